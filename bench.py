@@ -1,0 +1,353 @@
+"""Throughput of the ASD verifier step on GB300.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+
+Workload (one step = one asd_verify call, the whole hot path): the
+Qwen3-14B-shaped verify, B=32 requests x (K=8)+1 rows x V=151936 bf16 logits,
+gate 1.0, cap 2, budget 8.0 carried across steps. Inputs are resident in HBM,
+rotating over distinct logit buffers whose total exceeds 4x the L2 size, and the
+K timed steps replay CUDA graphs (one kernel node per step). Prints one JSON
+line (rank 0). Under torchrun each rank verifies its own batch (weak scaling, no
+collective on the data path; the barrier and the max over ranks time the job).
+
+--impl reference times the CPU oracle as it stands on the host cores (rank 0
+only), one full block of the same workload per step.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+METRIC = "verify rows/s & HBM GB/s (% of ~8 TB/s), V=151936 bf16 B=32 K=8"
+NOMINAL_HBM_GBS = 8000.0
+B, K, V = 32, 8, 151936
+GATE, CAP, BUDGET = 1.0, 2, 8.0
+WORKLOAD = "qwen3-14b-verify: B=32 requests, K=8 draft tokens (288 target rows), V=151936, bf16 logits, " \
+           "gate=1.0, cap=2, budget=8.0 carried across steps"
+KERNEL_SOURCE = os.path.join(ROOT, "paper_2608_03447_gb300", "csrc", "asd_verify.cu")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "verify_kernel_traffic.json")
+
+
+def peaks() -> dict:
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return {"hbm_gbs": float(p["hbm_gbs"]), "source": "measured"}
+    except (OSError, KeyError, ValueError):
+        return {"hbm_gbs": 6800.0, "source": "fallback"}
+
+
+def source_digest(path: str = KERNEL_SOURCE) -> str:
+    with open(path, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()
+
+
+def recorded_traffic() -> float | None:
+    """DRAM bytes per launch from the committed ncu summary, if it is for the current kernel source."""
+    try:
+        with open(TRAFFIC_FILE) as f:
+            rec = json.load(f)
+    except (OSError, ValueError):
+        return None
+    if rec.get("source_sha256") != source_digest():
+        return None
+    return float(rec["dram_bytes_per_launch"])
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling in the background (200 ms period)."""
+
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        self.proc = None
+        self.t0 = self.t1 = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.QUERY}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.file, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+
+    def mark_start(self):
+        self.t0 = time.time()
+
+    def mark_end(self):
+        self.t1 = time.time()
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.file.flush()
+        self.file.seek(0)
+        rows = [r.split(",") for r in self.file.read().strip().splitlines() if r.strip()]
+        os.unlink(self.file.name)
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            try:
+                sm.append(float(r[1]))
+                smax.append(float(r[2]))
+            except (ValueError, IndexError):
+                continue
+            for name, val in zip(names, r[5:9]):
+                if val.strip().lower() in ("active", "1"):
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def run_reference(args) -> None:
+    """The CPU oracle as it stands, on the host cores: one full block of the workload per step."""
+    import concurrent.futures as cf
+    from oracle import oracle
+    from paper_2608_03447_gb300 import inputs
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    cores = os.cpu_count() or 1
+    lib = oracle.load_library()
+    nblk = 2
+    blocks = [inputs.gen_block(B, K, V, torch.bfloat16, inputs.seed_for(1, 0, i), "cpu") for i in range(nblk)]
+    host = [(oracle.bf16_bits(b.logits), b.draft.numpy()) for b in blocks]
+    led = np.array([[BUDGET, 0.0]] * B, np.float32)
+
+    def one_request(args_):
+        z, x, b, led_b = args_
+        return oracle.verify(z[b:b + 1], x[b:b + 1], led_b, GATE, CAP, dtype=oracle.DTYPE_BF16, lib=lib)
+
+    pool = cf.ThreadPoolExecutor(max_workers=cores)
+
+    def step(i):
+        nonlocal led
+        z, x = host[i % nblk]
+        res = list(pool.map(one_request, [(z, x, b, led[b:b + 1]) for b in range(B)]))
+        led = np.concatenate([r["ledger"] for r in res])
+
+    for i in range(args.warmup):
+        step(i)
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        step(i)
+    dt = time.perf_counter() - t0
+    pool.shutdown()
+    rows_per_s = args.steps * B * (K + 1) / dt
+    line = {
+        "impl": "reference", "metric": METRIC, "value": rows_per_s, "unit": "rows/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "B": B, "K": K, "V": V, "l2": "host memory (CPU oracle)"},
+        "cpu_baseline": {"value": rows_per_s, "unit": "rows/s", "cores": cores, "kind": "oracle",
+                         "sample": f"{args.steps} full blocks of {B}x{K + 1}x{V} bf16, one request per thread"},
+        "e2e": {"value": rows_per_s, "unit": "rows/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def cpu_baseline(wl, seconds: float = 12.0) -> dict:
+    """The oracle as it stands on the host cores, on a bounded sample of the same workload."""
+    import concurrent.futures as cf
+    from oracle import oracle
+    lib = oracle.load_library()
+    cores = os.cpu_count() or 1
+    nblk = min(2, wl.nbuf)
+    host = [(oracle.bf16_bits(wl.logits[i].cpu()), wl.drafts[i].cpu().numpy()) for i in range(nblk)]
+    led = np.array([[BUDGET, 0.0]] * B, np.float32)
+
+    def one_request(a):
+        z, x, b = a
+        return oracle.verify(z[b:b + 1], x[b:b + 1], led[b:b + 1], GATE, CAP, dtype=oracle.DTYPE_BF16, lib=lib)
+
+    rows = 0
+    t0 = time.perf_counter()
+    with cf.ThreadPoolExecutor(max_workers=cores) as pool:
+        i = 0
+        while True:
+            z, x = host[i % nblk]
+            list(pool.map(one_request, [(z, x, b) for b in range(B)]))
+            rows += B * (K + 1)
+            i += 1
+            if time.perf_counter() - t0 >= seconds:
+                break
+    dt = time.perf_counter() - t0
+    return {"value": rows / dt, "unit": "rows/s", "cores": cores, "kind": "oracle",
+            "sample": f"{i} full blocks ({B}x{K + 1}x{V} bf16 from the GPU buffers), one request per thread, "
+                      f"{dt:.1f} s"}
+
+
+def run_gpu(args) -> None:
+    import torch.distributed as dist
+    from paper_2608_03447_gb300 import asd, inputs
+    from paper_2608_03447_gb300.workload import VerifyWorkload, l2_bytes
+
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+    asd.load()
+
+    wl = VerifyWorkload(B, K, V, torch.bfloat16, GATE, CAP, BUDGET, config=1 + 100 * rank, device=dev)
+    steps, warmup = args.steps, args.warmup
+    G = min(steps, 512)
+    graph_full = wl.capture(G, first=0)
+    graph_rem = wl.capture(steps % G, first=(steps // G) * G) if steps % G else None
+    wl.reset_ledger()
+    torch.cuda.synchronize(dev)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    clocks = ClockSampler(local)
+    clocks.start()
+    # warm-up: W graph replays, then untimed steps until ~1 s of load (clocks settle, sampler sees load)
+    stream = torch.cuda.current_stream(dev)
+    for _ in range(max(3, warmup)):
+        graph_full.replay()
+    t_soak = time.time()
+    while time.time() - t_soak < 1.0:
+        graph_full.replay()
+        torch.cuda.synchronize(dev)
+    barrier()
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks.mark_start()
+    start.record(stream)
+    for _ in range(steps // G):
+        graph_full.replay()
+    if graph_rem is not None:
+        graph_rem.replay()
+    end.record(stream)
+    end.synchronize()
+    barrier()
+    clocks.mark_end()
+    clk = clocks.stop()
+    ms = start.elapsed_time(end)
+    t = torch.tensor([ms], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    ms_max = float(t.item())
+    sec_per_step = ms_max / 1e3 / steps
+    rows_per_step = B * (K + 1)
+    value = world * rows_per_step / sec_per_step
+    bytes_per_launch = wl.bytes_per_step
+    achieved_gbs = bytes_per_launch / sec_per_step / 1e9
+
+    # end to end through the public API from pinned host buffers (copies inside the timed region)
+    e2e = run_e2e(wl, dev, steps=max(10, min(steps, 200)), world=world)
+
+    if rank == 0:
+        pk = peaks()
+        cpu = cpu_baseline(wl) if world == 1 else None
+        line = {
+            "metric": METRIC, "value": value, "unit": "rows/s", "n_gpus": world, "steps": steps,
+            "warmup": warmup, "ms_per_step": sec_per_step * 1e3, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "B": B, "K": K, "V": V, "gate": GATE, "cap": CAP,
+                       "budget": BUDGET, "parallelism": f"dp{world} (independent requests per rank)",
+                       "l2": f"inputs rotate over {wl.nbuf} logit buffers = "
+                             f"{wl.nbuf * bytes_per_launch / 1e6:.0f} MB (> 4x the {l2_bytes(dev) / 1e6:.0f} MB L2)",
+                       "launch": f"CUDA graphs of {G} steps, one kernel per step"},
+            "hbm_gbs": achieved_gbs, "pct_of_8tbs": achieved_gbs / NOMINAL_HBM_GBS,
+            "roofline": {"bound": "hbm", "achieved": achieved_gbs, "peak": pk["hbm_gbs"], "unit": "GB/s",
+                         "frac": achieved_gbs / pk["hbm_gbs"], "traffic": recorded_traffic(),
+                         "peak_source": pk["source"], "kernel": "verify_kernel<bf16, asd>",
+                         "algorithmic_bytes_per_launch": bytes_per_launch},
+            "clocks": clk,
+            "e2e": e2e,
+            "gpu_launches": steps,
+            "cpu_baseline": cpu,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def run_e2e(wl, dev, steps: int, world: int) -> dict:
+    """The same step through asd.verify_from_host: H2D of logits + drafts, verify, D2H of the results."""
+    from paper_2608_03447_gb300 import asd
+    import torch.distributed as dist
+    host_logits = [wl.logits[i].cpu().pin_memory() for i in range(2)]
+    host_draft = [wl.drafts[i].cpu().pin_memory() for i in range(2)]
+    dev_logits = torch.empty_like(wl.logits[0])
+    dev_draft = torch.empty_like(wl.drafts[0])
+    host_out = {k: torch.empty(v.shape, dtype=v.dtype, pin_memory=True)
+                for k, v in wl.out.items() if k in ("accepted_len", "committed", "recovery")}
+    stream = torch.cuda.current_stream(dev)
+    for i in range(3):
+        asd.verify_from_host(host_logits[i % 2], host_draft[i % 2], wl.ledger, GATE, CAP, dev_logits, dev_draft,
+                             wl.workspace, wl.out, host_out)
+    torch.cuda.synchronize(dev)
+    if world > 1:
+        dist.barrier()
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for i in range(steps):
+        asd.verify_from_host(host_logits[i % 2], host_draft[i % 2], wl.ledger, GATE, CAP, dev_logits, dev_draft,
+                             wl.workspace, wl.out, host_out)
+    end.record(stream)
+    end.synchronize()
+    ms = start.elapsed_time(end)
+    t = torch.tensor([ms], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    sec = float(t.item()) / 1e3
+    h2d = host_logits[0].numel() * host_logits[0].element_size() + host_draft[0].numel() * 4
+    d2h = sum(v.numel() * v.element_size() for v in host_out.values())
+    return {"value": world * steps * B * (K + 1) / sec, "unit": "rows/s", "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "steps": steps}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="asd", choices=["asd", "reference"])
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,133 @@
+/*
+ * asd.h - C ABI of libasd, the GB300 (sm_103a) verifier of Approximate
+ * Speculative Decoding (ASD, arXiv 2608.03447).
+ *
+ * One verifier step takes the target model's teacher-forced logits for a batch
+ * of draft blocks and, per request, returns the accepted prefix length, the
+ * committed tokens, the recovery (or bonus) token and the updated regret
+ * ledger (Sec. 3.2-3.3, Alg. 1).
+ *
+ * Conventions shared by every entry point
+ *   - Every array argument is DEVICE memory owned by the caller, contiguous,
+ *     row-major. The library allocates nothing and keeps no per-call state
+ *     outside the caller's workspace.
+ *   - Calls are asynchronous and ordered on `stream` (a cudaStream_t; NULL is
+ *     the legacy default stream). Nothing synchronises with the host.
+ *   - Indices are 0-based: request b in [0, B), draft position j in [0, K)
+ *     (the paper's i = j + 1), target row j in [0, K] (row K is the bonus row).
+ *   - A return value other than ASD_OK means that nothing was launched, except
+ *     ASD_ERR_CUDA, which reports a failed launch.
+ *   - Per-request data errors never abort the call: they set bits of
+ *     status[b] (ASD_STATUS_*). Such a request accepts nothing (a = 0), emits
+ *     y*_0 as its recovery token and keeps its ledger; for a NaN logit the
+ *     argmax is deterministic but unspecified.
+ *   - A workspace serves one call at a time: two calls that share a workspace
+ *     must be ordered on one stream (or otherwise serialised).
+ */
+#ifndef ASD_H
+#define ASD_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+struct CUstream_st;
+typedef struct CUstream_st* asd_stream_t; /* == cudaStream_t */
+
+/* The persistent per-request ledger (B, s) of Sec. 3.2: the request's total
+ * regret budget and the regret already spent in earlier rounds. budget = 0
+ * selects exact strict greedy verification (Alg. 1); budget = +INFINITY is
+ * allowed. Valid ledgers have 0 <= spent <= budget and no NaN. */
+typedef struct {
+  float budget;
+  float spent;
+} asd_ledger;
+
+/* Logit storage types. */
+enum { ASD_F32 = 0, ASD_BF16 = 1 };
+
+/* Return codes. */
+enum {
+  ASD_OK = 0,
+  ASD_ERR_NULL = 1,      /* a required pointer is NULL */
+  ASD_ERR_SHAPE = 2,     /* B < 0, K < 0, K > 31, V < 1, or H invalid */
+  ASD_ERR_DTYPE = 3,     /* unknown dtype code */
+  ASD_ERR_CONTROL = 4,   /* gate < 0 or NaN, cap < 0 */
+  ASD_ERR_WORKSPACE = 5, /* workspace smaller than the size query returns */
+  ASD_ERR_ALIGN = 6,     /* pointer not aligned as documented */
+  ASD_ERR_CUDA = 7,      /* a CUDA call failed (launch or device query) */
+  ASD_ERR_DEVICE = 8     /* the current device cannot run the kernel (not sm_103) */
+};
+
+/* Per-request status bits (status[b]). */
+#define ASD_STATUS_DRAFT_RANGE 1u /* a draft id outside [0, V) */
+#define ASD_STATUS_NAN_LOGIT 2u   /* a NaN among the request's K+1 logit rows */
+#define ASD_STATUS_BAD_LEDGER 4u  /* budget < 0 or NaN, spent < 0 or NaN, spent > budget */
+
+/* Largest draft length: one warp lane per target row of a block. */
+#define ASD_MAX_K 31
+
+/* Bytes of workspace that asd_verify / asd_verify_strict need for (B, K, V,
+ * dtype). Writes *bytes; returns ASD_ERR_SHAPE / ASD_ERR_DTYPE / ASD_ERR_NULL
+ * on bad arguments. */
+int asd_workspace_size(int B, int K, int V, int dtype, size_t* bytes);
+
+/* Zero a workspace (cudaMemsetAsync on `stream`). Required once before the
+ * first call that uses it; every verify call leaves the workspace zeroed again
+ * when it completes, so it can be reused (and captured in a CUDA graph) with
+ * no further initialisation. */
+int asd_workspace_init(void* workspace, size_t bytes, asd_stream_t stream);
+
+/*
+ * ASD verification of B draft blocks (Eq. 1, 3, 5-13; Alg. 1).
+ *
+ * logits        [B, K+1, V], dtype ASD_F32 or ASD_BF16; row b*(K+1)+j holds
+ *               z_{j+1}. Aligned to its element size; any further alignment
+ *               is handled.
+ * draft         [B, K] int32 draft tokens x (may be NULL when K = 0)
+ * ledger        [B] in/out. spent is updated to s' = fl(s + C_a) (Eq. 13);
+ *               left untouched when budget == 0 or the request is flagged.
+ * gate          g of Eq. 7 (>= 0; +INFINITY disables the gate)
+ * cap           M of Eq. 10 (>= 0; INT32_MAX disables the cap)
+ * accepted_len  [B]       a = longest feasible prefix (Eq. 12)
+ * committed     [B, K+1]  x_0..x_{a-1}, y*_a, then -1 padding
+ * recovery      [B]       y*_a: the recovery token (a < K) or the bonus (a = K)
+ * row_argmax    [B, K+1]  y*_j (lowest index on ties); may be NULL
+ * row_regret    [B, K]    r_j = fl32(z_j(y*_j) - z_j(x_j)), NaN for an
+ *                         out-of-range draft; may be NULL
+ * status        [B]       ASD_STATUS_* bits; may be NULL
+ * workspace     >= asd_workspace_size(...) bytes, 16-byte aligned, zeroed
+ *               by asd_workspace_init before first use
+ *
+ * Arithmetic (all fp32, round to nearest): argmax by IEEE comparison
+ * (-0 == +0), then per request, left to right over the mismatches d_j = 1:
+ * C' = C + r_j; accept while r_j / (K - j) <= g, fl(s + C') <= budget and
+ * N' <= M; a is the first position that fails (else K). budget == 0
+ * dispatches to the strict rule (Eq. 2) and keeps the ledger.
+ */
+int asd_verify(const void* logits, int dtype, int B, int K, int V, const int32_t* draft,
+               asd_ledger* ledger, float gate, int cap, int32_t* accepted_len,
+               int32_t* committed, int32_t* recovery, int32_t* row_argmax, float* row_regret,
+               int32_t* status, void* workspace, size_t workspace_bytes, asd_stream_t stream);
+
+/*
+ * Strict greedy verification (Eq. 2): a = the first j with x_j != y*_j (else
+ * K); committed and recovery as in asd_verify (the bonus y*_K is appended when
+ * a = K). No ledger. Same arguments, layouts and workspace as asd_verify.
+ */
+int asd_verify_strict(const void* logits, int dtype, int B, int K, int V, const int32_t* draft,
+                      int32_t* accepted_len, int32_t* committed, int32_t* recovery,
+                      int32_t* row_argmax, float* row_regret, int32_t* status, void* workspace,
+                      size_t workspace_bytes, asd_stream_t stream);
+
+/* Human-readable text of a return code. Never NULL. */
+const char* asd_status_string(int code);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ASD_H */

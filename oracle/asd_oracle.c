@@ -134,6 +134,40 @@ static int ledger_invalid(float budget, float spent) {
 }
 
 /*
+ * Alg. 1 for one request, given its row-stage results: y*_0..y*_K, the
+ * regrets r_0..r_{K-1} and the row-stage status bits (NaN logit, draft range).
+ * Writes a, the committed tokens, the recovery token and the status word, and
+ * updates the ledger (budget, spent) unless strict, zero-budget or flagged.
+ */
+static void select_block(int K, const int32_t* x, const int32_t* y, const float* r, int flags,
+                         float* ledger_b, float gate, int cap, int strict, int32_t* accepted_len_b,
+                         int32_t* committed_b, int32_t* recovery_b, int32_t* status_b) {
+  float budget = ledger_b[0];
+  float spent = ledger_b[1];
+  if (!strict && ledger_invalid(budget, spent)) flags |= ORC_STATUS_BAD_LEDGER;
+
+  int a;
+  if (flags) {
+    a = 0; /* a flagged request accepts nothing and keeps its ledger */
+  } else if (strict || budget == 0.0f) {
+    a = strict_prefix(K, x, y); /* Alg. 1: B = 0 -> exact greedy output, state kept */
+  } else {
+    float C = 0.0f;
+    a = asd_prefix(K, x, y, r, budget, spent, gate, cap, &C);
+    ledger_b[1] = spent + C; /* Eq. 13 */
+  }
+  *accepted_len_b = a;
+  *recovery_b = y[a]; /* y*_{a+1}: recovery if a < K, bonus if a = K */
+  for (int j = 0; j <= K; j++) {
+    int32_t token = -1;
+    if (j < a) token = x[j];
+    else if (j == a) token = y[a];
+    committed_b[j] = token;
+  }
+  *status_b = flags;
+}
+
+/*
  * Verify B draft blocks.
  *   logits       [B, K+1, V] fp32 or bf16 bits, row-major
  *   draft        [B, K] int32
@@ -176,29 +210,27 @@ int oracle_verify(const void* logits, int dtype, int B, int K, int V, const int3
       }
       row_regret[(int64_t)b * K + j] = r[j];
     }
-    float budget = ledger[2 * b];
-    float spent = ledger[2 * b + 1];
-    if (!strict && ledger_invalid(budget, spent)) flags |= ORC_STATUS_BAD_LEDGER;
+    select_block(K, x, y, r, flags, ledger + 2 * b, gate, cap, strict, accepted_len + b,
+                 committed + (int64_t)b * (K + 1), recovery + b, status + b);
+  }
+  return 0;
+}
 
-    int a;
-    if (flags) {
-      a = 0; /* a flagged request accepts nothing and keeps its ledger */
-    } else if (strict || budget == 0.0f) {
-      a = strict_prefix(K, x, y); /* Alg. 1: B = 0 -> exact greedy output, state kept */
-    } else {
-      float C = 0.0f;
-      a = asd_prefix(K, x, y, r, budget, spent, gate, cap, &C);
-      ledger[2 * b + 1] = spent + C; /* Eq. 13 */
-    }
-    accepted_len[b] = a;
-    recovery[b] = y[a]; /* y*_{a+1}: recovery if a < K, bonus if a = K */
-    for (int j = 0; j <= K; j++) {
-      int32_t token = -1;
-      if (j < a) token = x[j];
-      else if (j == a) token = y[a];
-      committed[(int64_t)b * (K + 1) + j] = token;
-    }
-    status[b] = flags;
+/*
+ * The selection stage alone (Alg. 1 after Eq. 1 and Eq. 3), for callers that
+ * already hold the row-stage results of a block (row_argmax [B, K+1],
+ * row_regret [B, K], row_status [B] = the status bits of a strict run) and
+ * want to replay the selection under other controls.
+ */
+int oracle_select(int B, int K, const int32_t* draft, const int32_t* row_argmax_in,
+                  const float* row_regret_in, const int32_t* row_status, float* ledger,
+                  float gate, int cap, int strict, int32_t* accepted_len, int32_t* committed,
+                  int32_t* recovery, int32_t* status) {
+  if (B < 0 || K < 0 || K > 31) return -1;
+  for (int b = 0; b < B; b++) {
+    select_block(K, draft + (int64_t)b * K, row_argmax_in + (int64_t)b * (K + 1),
+                 row_regret_in + (int64_t)b * K, row_status[b], ledger + 2 * b, gate, cap, strict,
+                 accepted_len + b, committed + (int64_t)b * (K + 1), recovery + b, status + b);
   }
   return 0;
 }

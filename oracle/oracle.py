@@ -48,6 +48,8 @@ def _bind(lib: ctypes.CDLL) -> ctypes.CDLL:
     lib.oracle_verify.restype = i32
     lib.oracle_verify.argtypes = [vp, i32, i32, i32, i32, vp, vp, f32, i32, i32,
                                   vp, vp, vp, vp, vp, vp]
+    lib.oracle_select.restype = i32
+    lib.oracle_select.argtypes = [i32, i32, vp, vp, vp, vp, vp, f32, i32, i32, vp, vp, vp, vp]
     lib.oracle_lmhead_logits.restype = None
     lib.oracle_lmhead_logits.argtypes = [vp, vp, i32, i32, vp, i32, vp, vp]
     return lib
@@ -138,6 +140,32 @@ def verify(logits, draft, ledger=None, gate: float = 1.0, cap: int = 2, strict: 
                            _ptr(out["row_regret"]), _ptr(out["status"]))
     if rc != 0:
         raise ValueError(f"oracle_verify rejected its arguments (B={B}, K={K}, V={V})")
+    out["ledger"] = led
+    return out
+
+
+def select(draft, row_argmax, row_regret, row_status, ledger, gate: float, cap: int,
+           strict: bool = False, lib: ctypes.CDLL | None = None) -> dict:
+    """Alg. 1 alone, replayed on the row-stage results of an earlier (strict) oracle run."""
+    lib = lib or load_library()
+    y = np.ascontiguousarray(row_argmax, dtype=np.int32)
+    B, K1 = y.shape
+    K = K1 - 1
+    x = np.ascontiguousarray(draft, dtype=np.int32).reshape(B, K)
+    r = np.ascontiguousarray(row_regret, dtype=np.float32).reshape(B, K)
+    st_in = np.ascontiguousarray(row_status, dtype=np.int32).reshape(B)
+    led = np.array(np.asarray(ledger, dtype=np.float32).reshape(B, 2), copy=True)
+    out = {
+        "accepted_len": np.zeros(B, np.int32),
+        "committed": np.zeros((B, K1), np.int32),
+        "recovery": np.zeros(B, np.int32),
+        "status": np.zeros(B, np.int32),
+    }
+    rc = lib.oracle_select(B, K, _ptr(x), _ptr(y), _ptr(r), _ptr(st_in), _ptr(led), float(gate), int(cap),
+                           1 if strict else 0, _ptr(out["accepted_len"]), _ptr(out["committed"]),
+                           _ptr(out["recovery"]), _ptr(out["status"]))
+    if rc != 0:
+        raise ValueError("oracle_select rejected its arguments")
     out["ledger"] = led
     return out
 

@@ -1,0 +1,210 @@
+"""ctypes binding of libasd (include/asd.h): argument marshalling only.
+
+Every step of the verifier runs in the library's CUDA kernels; this module
+turns torch tensors into device pointers, passes torch's current CUDA stream,
+and raises on a non-zero return code. There is no fallback: if libasd.so is
+missing the first call raises.
+
+Entry points mirror the C names: ``verify`` (asd_verify), ``verify_strict``
+(asd_verify_strict), ``workspace_size``, ``workspace_init``, ``status_string``.
+Ledgers are float32 tensors of shape [B, 2] holding (budget, spent), the
+memory layout of ``asd_ledger``.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+import threading
+
+import torch
+
+PKG = os.path.dirname(os.path.abspath(__file__))
+LIBRARY = os.path.join(PKG, "libasd.so")
+HEADER = os.path.join(os.path.dirname(PKG), "include", "asd.h")
+
+F32 = 0
+BF16 = 1
+
+OK = 0
+STATUS_DRAFT_RANGE = 1
+STATUS_NAN_LOGIT = 2
+STATUS_BAD_LEDGER = 4
+MAX_K = 31
+INT32_MAX = 2**31 - 1
+
+_lock = threading.Lock()
+_lib = None
+
+
+class AsdError(RuntimeError):
+    def __init__(self, fn: str, code: int):
+        self.code = code
+        super().__init__(f"{fn} returned {code}: {status_string(code) if _lib else code}")
+
+
+def _declare(lib: ctypes.CDLL) -> ctypes.CDLL:
+    vp, i32, f32, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_float, ctypes.c_size_t
+    lib.asd_workspace_size.argtypes = [i32, i32, i32, i32, ctypes.POINTER(sz)]
+    lib.asd_workspace_size.restype = i32
+    lib.asd_workspace_init.argtypes = [vp, sz, vp]
+    lib.asd_workspace_init.restype = i32
+    lib.asd_verify.argtypes = [vp, i32, i32, i32, i32, vp, vp, f32, i32, vp, vp, vp, vp, vp, vp, vp, sz, vp]
+    lib.asd_verify.restype = i32
+    lib.asd_verify_strict.argtypes = [vp, i32, i32, i32, i32, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
+    lib.asd_verify_strict.restype = i32
+    lib.asd_status_string.argtypes = [i32]
+    lib.asd_status_string.restype = ctypes.c_char_p
+    if hasattr(lib, "asd_lmhead_workspace_size"):
+        lib.asd_lmhead_workspace_size.argtypes = [i32, i32, i32, i32, ctypes.POINTER(sz)]
+        lib.asd_lmhead_workspace_size.restype = i32
+        lib.asd_lmhead_verify.argtypes = [vp, vp, i32, i32, i32, i32, vp, vp, f32, i32,
+                                          vp, vp, vp, vp, vp, vp, vp, sz, vp]
+        lib.asd_lmhead_verify.restype = i32
+    return lib
+
+
+def load(path: str = LIBRARY) -> ctypes.CDLL:
+    """Open libasd.so (once). Raises if it has not been built."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(path):
+                raise RuntimeError(f"{path} is missing: build it with __graft_entry__.build() "
+                                   "(python -m paper_2608_03447_gb300.build)")
+            _lib = _declare(ctypes.CDLL(path))
+    return _lib
+
+
+def declared_functions(header: str = HEADER) -> list[str]:
+    """Names of the functions that include/asd.h declares."""
+    with open(header) as f:
+        text = f.read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(asd_[a-z0-9_]+)\s*\(", text)))
+
+
+def status_string(code: int) -> str:
+    return load().asd_status_string(int(code)).decode()
+
+
+def _check(fn: str, rc: int) -> None:
+    if rc != OK:
+        raise AsdError(fn, rc)
+
+
+def _ptr(t: torch.Tensor | None) -> int | None:
+    if t is None:
+        return None
+    return t.data_ptr()
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.float32:
+        return F32
+    if t.dtype == torch.bfloat16:
+        return BF16
+    raise TypeError(f"logits must be float32 or bfloat16, got {t.dtype}")
+
+
+def workspace_size(B: int, K: int, V: int, dtype: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check("asd_workspace_size", load().asd_workspace_size(B, K, V, dtype, ctypes.byref(n)))
+    return n.value
+
+
+class Workspace:
+    """Device scratch for one stream of verify calls; zeroed once at creation."""
+
+    def __init__(self, B: int, K: int, V: int, dtype: int, device=None, stream=None):
+        self.nbytes = workspace_size(B, K, V, dtype)
+        self.buffer = torch.empty(self.nbytes, dtype=torch.uint8, device=device or "cuda")
+        _check("asd_workspace_init", load().asd_workspace_init(self.buffer.data_ptr(), self.nbytes, _stream(stream)))
+
+    @property
+    def ptr(self) -> int:
+        return self.buffer.data_ptr()
+
+
+def make_ledger(B: int, budget: float, spent: float = 0.0, device="cuda") -> torch.Tensor:
+    led = torch.empty(B, 2, dtype=torch.float32, device=device)
+    led[:, 0] = budget
+    led[:, 1] = spent
+    return led
+
+
+def alloc_outputs(B: int, K: int, device="cuda", with_rows: bool = True) -> dict:
+    out = {
+        "accepted_len": torch.empty(B, dtype=torch.int32, device=device),
+        "committed": torch.empty(B, K + 1, dtype=torch.int32, device=device),
+        "recovery": torch.empty(B, dtype=torch.int32, device=device),
+        "status": torch.empty(B, dtype=torch.int32, device=device),
+    }
+    if with_rows:
+        out["row_argmax"] = torch.empty(B, K + 1, dtype=torch.int32, device=device)
+        out["row_regret"] = torch.empty(B, K, dtype=torch.float32, device=device)
+    return out
+
+
+def _shape(logits: torch.Tensor, draft: torch.Tensor):
+    if logits.dim() != 3 or not logits.is_cuda or not logits.is_contiguous():
+        raise ValueError("logits must be a contiguous CUDA tensor [B, K+1, V]")
+    B, K1, V = logits.shape
+    K = K1 - 1
+    if draft.shape != (B, K) or draft.dtype != torch.int32 or not draft.is_contiguous():
+        raise ValueError("draft must be a contiguous int32 tensor [B, K]")
+    return B, K, V
+
+
+def verify(logits: torch.Tensor, draft: torch.Tensor, ledger: torch.Tensor, gate: float, cap: int,
+           workspace: Workspace | None = None, out: dict | None = None, stream=None) -> dict:
+    """asd_verify: ASD verification of a batch of draft blocks; updates ``ledger`` in place."""
+    B, K, V = _shape(logits, draft)
+    if ledger.shape != (B, 2) or ledger.dtype != torch.float32 or not ledger.is_contiguous():
+        raise ValueError("ledger must be a contiguous float32 tensor [B, 2] of (budget, spent)")
+    code = _dtype_code(logits)
+    ws = workspace or Workspace(B, K, V, code, logits.device, stream)
+    o = out or alloc_outputs(B, K, logits.device)
+    rc = load().asd_verify(_ptr(logits), code, B, K, V, _ptr(draft), _ptr(ledger), float(gate), int(cap),
+                           _ptr(o["accepted_len"]), _ptr(o["committed"]), _ptr(o["recovery"]),
+                           _ptr(o.get("row_argmax")), _ptr(o.get("row_regret")), _ptr(o.get("status")),
+                           ws.ptr, ws.nbytes, _stream(stream))
+    _check("asd_verify", rc)
+    return o
+
+
+def verify_strict(logits: torch.Tensor, draft: torch.Tensor, workspace: Workspace | None = None,
+                  out: dict | None = None, stream=None) -> dict:
+    """asd_verify_strict: strict greedy verification (Eq. 2)."""
+    B, K, V = _shape(logits, draft)
+    code = _dtype_code(logits)
+    ws = workspace or Workspace(B, K, V, code, logits.device, stream)
+    o = out or alloc_outputs(B, K, logits.device)
+    rc = load().asd_verify_strict(_ptr(logits), code, B, K, V, _ptr(draft),
+                                  _ptr(o["accepted_len"]), _ptr(o["committed"]), _ptr(o["recovery"]),
+                                  _ptr(o.get("row_argmax")), _ptr(o.get("row_regret")), _ptr(o.get("status")),
+                                  ws.ptr, ws.nbytes, _stream(stream))
+    _check("asd_verify_strict", rc)
+    return o
+
+
+def verify_from_host(logits_host: torch.Tensor, draft_host: torch.Tensor, ledger: torch.Tensor, gate: float,
+                     cap: int, logits_dev: torch.Tensor, draft_dev: torch.Tensor, workspace: Workspace,
+                     out: dict, host_out: dict, stream=None) -> dict:
+    """End-to-end step from pinned host buffers: copy in, verify, copy the per-request results out.
+
+    The ledger stays on the device (it is the request state carried between
+    rounds); the copies are asynchronous on ``stream``.
+    """
+    logits_dev.copy_(logits_host, non_blocking=True)
+    draft_dev.copy_(draft_host, non_blocking=True)
+    verify(logits_dev, draft_dev, ledger, gate, cap, workspace, out, stream)
+    for k in ("accepted_len", "committed", "recovery"):
+        host_out[k].copy_(out[k], non_blocking=True)
+    return host_out

@@ -321,9 +321,25 @@ def pin_lmhead_vs_numpy(lib):
     assert np.array_equal(z32, z64.astype(np.float32))
 
 
+def pin_select_replays_verify(lib):
+    """The selection-only entry on a strict run's row results == the full verify, for every control."""
+    import torch
+    from paper_2608_03447_gb300 import inputs
+    block = inputs.gen_block(8, 6, 700, torch.float32, 777)
+    z, x = block.logits.numpy(), block.draft.numpy()
+    x[3, 2] = 700                                  # one out-of-range draft
+    rows = oracle.verify(z, x, None, strict=True, lib=lib)
+    for g, M, bud, s in ((1.0, 2, 4.0, 0.5), (0.25, 1, 8.0, 0.0), (math.inf, INT32_MAX, 0.0, 0.0), (2.0, 4, 1.0, 2.0)):
+        led = np.array([[bud, s]] * 8, np.float32)
+        full = oracle.verify(z, x, led, g, M, lib=lib)
+        sel = oracle.select(x, rows["row_argmax"], rows["row_regret"], rows["status"], led, g, M, lib=lib)
+        for key in ("accepted_len", "committed", "recovery", "status", "ledger"):
+            assert np.array_equal(full[key], sel[key]), key
+
+
 ALL_PINS = [pin_argmax_vs_numpy, pin_regret_vs_gather, pin_selection_bruteforce, pin_zero_budget_is_strict,
             pin_gate_and_budget_boundaries, pin_fig1, pin_cap_zero_is_strict, pin_carry_ledger,
-            pin_status_flags, pin_lmhead_vs_numpy]
+            pin_status_flags, pin_lmhead_vs_numpy, pin_select_replays_verify]
 
 
 def run_all(lib, quick=False):

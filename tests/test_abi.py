@@ -1,0 +1,104 @@
+"""The C ABI on the host: the library loads, exports every declared symbol, and rejects bad
+arguments before touching CUDA (so these run without a GPU)."""
+import ctypes
+import math
+import os
+
+import pytest
+
+from paper_2608_03447_gb300 import asd, build
+
+NULL = None
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if not os.path.exists(asd.LIBRARY) or any(
+            os.path.getmtime(s) > os.path.getmtime(asd.LIBRARY) for s in build.sources()):
+        build.build()
+    return asd.load()
+
+
+def test_every_declared_symbol_is_exported(lib):
+    declared = asd.declared_functions()
+    assert {"asd_verify", "asd_verify_strict", "asd_workspace_size", "asd_workspace_init",
+            "asd_status_string"} <= set(declared)
+    for name in declared:
+        assert hasattr(lib, name), f"{name} is declared in include/asd.h but not exported"
+
+
+def test_status_strings(lib):
+    for code in range(0, 9):
+        assert asd.status_string(code)
+    assert asd.status_string(12345) == "unknown status code"
+
+
+def test_workspace_size(lib):
+    n = asd.workspace_size(32, 8, 151936, asd.BF16)
+    assert n >= 32 * 9 * 12 + 32 * 12 and n % 256 == 0
+    n0 = asd.workspace_size(0, 8, 10, asd.F32)
+    assert n0 > 0
+    sz = ctypes.c_size_t(0)
+    assert lib.asd_workspace_size(1, 32, 10, asd.F32, ctypes.byref(sz)) == 2   # K > 31
+    assert lib.asd_workspace_size(1, -1, 10, asd.F32, ctypes.byref(sz)) == 2
+    assert lib.asd_workspace_size(1, 4, 0, asd.F32, ctypes.byref(sz)) == 2     # V < 1
+    assert lib.asd_workspace_size(1, 4, 10, 7, ctypes.byref(sz)) == 3          # dtype
+    assert lib.asd_workspace_size(1, 4, 10, asd.F32, None) == 1
+
+
+def _verify(lib, **kw):
+    a = dict(logits=0x1000, dtype=asd.F32, B=2, K=3, V=10, draft=0x2000, ledger=0x3000, gate=1.0, cap=2,
+             acc=0x4000, com=0x5000, rec=0x6000, ya=NULL, rr=NULL, st=NULL, ws=0x7000, wsb=1 << 20)
+    a.update(kw)
+    return lib.asd_verify(a["logits"], a["dtype"], a["B"], a["K"], a["V"], a["draft"], a["ledger"], a["gate"],
+                          a["cap"], a["acc"], a["com"], a["rec"], a["ya"], a["rr"], a["st"], a["ws"], a["wsb"], None)
+
+
+def test_verify_rejects_bad_arguments_without_launching(lib):
+    # fake (never dereferenced) pointers: every case returns before any CUDA call
+    assert _verify(lib, dtype=5) == 3
+    assert _verify(lib, K=32) == 2
+    assert _verify(lib, V=0) == 2
+    assert _verify(lib, B=-1) == 2
+    assert _verify(lib, logits=NULL) == 1
+    assert _verify(lib, draft=NULL) == 1
+    assert _verify(lib, ledger=NULL) == 1
+    assert _verify(lib, acc=NULL) == 1
+    assert _verify(lib, ws=NULL) == 1
+    assert _verify(lib, gate=-0.5) == 4
+    assert _verify(lib, gate=math.nan) == 4
+    assert _verify(lib, cap=-1) == 4
+    assert _verify(lib, wsb=16) == 5
+    assert _verify(lib, ws=0x7004) == 6                      # workspace not 16-byte aligned
+    assert _verify(lib, logits=0x1001) == 6                  # fp32 logits not 4-byte aligned
+    assert _verify(lib, dtype=asd.BF16, logits=0x1001) == 6  # bf16 logits not 2-byte aligned
+    assert _verify(lib, B=0) == 0                            # empty batch: nothing to do
+
+
+def test_strict_rejects_bad_arguments(lib):
+    def strict(**kw):
+        a = dict(logits=0x1000, dtype=asd.F32, B=2, K=3, V=10, draft=0x2000, acc=0x4000, com=0x5000,
+                 rec=0x6000, ws=0x7000, wsb=1 << 20)
+        a.update(kw)
+        return lib.asd_verify_strict(a["logits"], a["dtype"], a["B"], a["K"], a["V"], a["draft"], a["acc"],
+                                     a["com"], a["rec"], None, None, None, a["ws"], a["wsb"], None)
+    assert strict(draft=NULL) == 1
+    assert strict(K=0, draft=NULL, B=0) == 0
+    assert strict(K=40) == 2
+    assert strict(wsb=0) == 5
+
+
+def test_workspace_init_null(lib):
+    assert lib.asd_workspace_init(None, 256, None) == 1
+
+
+def test_binding_fails_loudly_without_library(tmp_path):
+    with pytest.raises(RuntimeError):
+        asd._declare  # the module is importable without the library
+        import importlib
+        mod = importlib.reload(asd)
+        try:
+            mod._lib = None
+            mod.load(str(tmp_path / "missing.so"))
+        finally:
+            importlib.reload(asd)

@@ -55,6 +55,10 @@ def test_lmhead_fp64_matches_numpy(oracle_lib):
     P.pin_lmhead_vs_numpy(oracle_lib)
 
 
+def test_select_replays_verify(oracle_lib):
+    P.pin_select_replays_verify(oracle_lib)
+
+
 def test_k_zero_emits_bonus_only(oracle_lib):
     """K = 0 (no draft tokens): a = 0 = K, and the only emitted token is the bonus y*_1."""
     z = np.zeros((3, 1, 5), np.float32)
@@ -155,8 +159,8 @@ MUTANTS = {
     "cumulative regret not accumulated": ("float C_next = C + r[j];", "float C_next = r[j];"),
     "matches treated as exceptions": ("if (x[j] == y[j]) continue; /* d = 0 */", ""),
     "no zero-budget dispatch": ("} else if (strict || budget == 0.0f) {", "} else if (strict) {"),
-    "ledger not updated": ("ledger[2 * b + 1] = spent + C; /* Eq. 13 */", ""),
-    "recovery from the previous row": ("recovery[b] = y[a];", "recovery[b] = y[a > 0 ? a - 1 : 0];"),
+    "ledger not updated": ("ledger_b[1] = spent + C; /* Eq. 13 */", ""),
+    "recovery from the previous row": ("*recovery_b = y[a];", "*recovery_b = y[a > 0 ? a - 1 : 0];"),
     "committed keeps the mismatched draft": ("if (j < a) token = x[j];", "if (j <= a) token = x[j];"),
     "strict stops one late": ("if (x[j] != y[j]) return j;", "if (x[j] != y[j]) return j + 1;"),
     "lm-head accumulates in fp32": ("double acc = 0.0;", "float acc = 0.0f;"),

@@ -1,0 +1,275 @@
+"""Parity of the CUDA verifier (asd_verify / asd_verify_strict) with the CPU oracle.
+
+Bit-exact on every output: argmax indices, accepted lengths, committed and
+recovery tokens, status words, and the fp32 regrets and ledgers (same fp32
+operation order on both sides). Requests flagged for a NaN logit are compared
+on what is specified for them (status, a = 0, ledger kept).
+"""
+import concurrent.futures as cf
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import oracle
+from paper_2608_03447_gb300 import inputs
+
+pytestmark = pytest.mark.gpu
+INT32_MAX = 2**31 - 1
+
+
+def _np(out: dict) -> dict:
+    return {k: v.cpu().numpy() for k, v in out.items()}
+
+
+def gpu_verify(asd, logits, draft, ledger, gate, cap, strict=False):
+    if strict:
+        out = asd.verify_strict(logits, draft)
+    else:
+        out = asd.verify(logits, draft, ledger, gate, cap)
+    torch.cuda.synchronize()
+    res = _np(out)
+    if ledger is not None:
+        res["ledger"] = ledger.cpu().numpy()
+    return res
+
+
+def assert_parity(gpu: dict, orc: dict, what: str = "", ledger: bool = True):
+    st = orc["status"]
+    assert np.array_equal(gpu["status"], st), f"{what}: status"
+    ok = (st & oracle.STATUS_NAN_LOGIT) == 0   # NaN rows: the argmax is unspecified
+    for key in ("accepted_len", "recovery"):
+        assert np.array_equal(gpu[key][ok], orc[key][ok]), f"{what}: {key}"
+    for key in ("committed", "row_argmax"):
+        if key in gpu:
+            diff = np.argwhere(gpu[key][ok] != orc[key][ok])
+            assert diff.size == 0, f"{what}: {key} differs at {diff[:5].tolist()}"
+    if "row_regret" in gpu:
+        g, o = gpu["row_regret"][ok], orc["row_regret"][ok]
+        same = (g.view(np.uint32) == o.view(np.uint32)) | (np.isnan(g) & np.isnan(o))
+        assert same.all(), f"{what}: row_regret differs at {np.argwhere(~same)[:5].tolist()}"
+    assert np.array_equal(gpu["accepted_len"][~ok], np.zeros((~ok).sum(), np.int32))
+    if ledger:
+        assert np.array_equal(gpu["ledger"].view(np.uint32), orc["ledger"].view(np.uint32)), f"{what}: ledger"
+
+
+def run_sequence(asd, B, K, V, dtype, blocks, gate, cap, budget, config, mix=inputs.MIX_DEFAULT, point=0):
+    """Sequential blocks on the same requests; the GPU carries its ledger on the device."""
+    led_gpu = asd.make_ledger(B, budget)
+    led_orc = np.array([[budget, 0.0]] * B, np.float32)
+    for blk in blocks:
+        b = inputs.gen_block(B, K, V, dtype, inputs.seed_for(config, point, blk), "cuda", mix=mix)
+        g = gpu_verify(asd, b.logits, b.draft, led_gpu, gate, cap)
+        o = oracle.verify(b.logits.cpu(), b.draft.cpu().numpy(), led_orc, gate, cap)
+        assert_parity(g, o, f"config {config} block {blk}")
+        led_orc = o["ledger"]
+        # strict entry on the same block
+        gs = gpu_verify(asd, b.logits, b.draft, None, 0, 0, strict=True)
+        os_ = oracle.verify(b.logits.cpu(), b.draft.cpu().numpy(), None, strict=True)
+        assert_parity(gs, os_, f"config {config} block {blk} strict", ledger=False)
+    return led_orc
+
+
+def test_tiny_fp32_sixteen_blocks(asd):
+    cfg = inputs.CONFIGS[0]
+    led = run_sequence(asd, cfg["B"], cfg["K"], cfg["V"], cfg["dtype"], range(cfg["blocks"]),
+                       cfg["gate"], cfg["cap"], cfg["budget"], 0)
+    assert np.all(led[:, 1] <= cfg["budget"])
+
+
+def test_tiny_zero_budget_is_strict(asd):
+    cfg = inputs.CONFIGS[0]
+    B, K, V = cfg["B"], cfg["K"], cfg["V"]
+    for blk in range(cfg["blocks"]):
+        b = inputs.gen_block(B, K, V, cfg["dtype"], inputs.seed_for(0, 1, blk), "cuda")
+        led = asd.make_ledger(B, 0.0)
+        g = gpu_verify(asd, b.logits, b.draft, led, cfg["gate"], cfg["cap"])
+        s = gpu_verify(asd, b.logits, b.draft, None, 0, 0, strict=True)
+        for key in ("accepted_len", "committed", "recovery", "row_argmax", "status"):
+            assert np.array_equal(g[key], s[key]), key
+        assert np.array_equal(g["ledger"], np.zeros((B, 2), np.float32))
+
+
+def test_qwen3_shape_bf16_blocks(asd):
+    cfg = inputs.CONFIGS[1]
+    run_sequence(asd, cfg["B"], cfg["K"], cfg["V"], cfg["dtype"], range(8), cfg["gate"], cfg["cap"],
+                 cfg["budget"], 1)
+
+
+def test_budget_cap_sweep(asd):
+    """B=128, K=16, V=151936 bf16: 64 control points x 16 sequential blocks, ledger reset per point."""
+    cfg = inputs.CONFIGS[2]
+    B, K, V = cfg["B"], cfg["K"], cfg["V"]
+    nblocks = cfg["blocks"]
+    blocks, rows = [], []
+    for blk in range(nblocks):
+        b = inputs.gen_block(B, K, V, cfg["dtype"], inputs.seed_for(2, 0, blk), "cuda")
+        blocks.append(b)
+        rows.append(oracle.verify(b.logits.cpu(), b.draft.cpu().numpy(), None, strict=True))
+    for g in cfg["gates"]:
+        for M in cfg["caps"]:
+            for bud in cfg["budgets"]:
+                led_gpu = asd.make_ledger(B, bud)
+                led_orc = np.array([[bud, 0.0]] * B, np.float32)
+                for blk in range(nblocks):
+                    b, r = blocks[blk], rows[blk]
+                    out = gpu_verify(asd, b.logits, b.draft, led_gpu, g, M)
+                    o = oracle.select(b.draft.cpu().numpy(), r["row_argmax"], r["row_regret"], r["status"],
+                                      led_orc, g, M)
+                    o["row_argmax"], o["row_regret"] = r["row_argmax"], r["row_regret"]
+                    assert_parity(out, o, f"g={g} M={M} B={bud} block {blk}")
+                    led_orc = o["ledger"]
+                    if bud == 0.0:
+                        assert np.array_equal(out["committed"], r["committed"]), "budget 0 != strict"
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+def test_large_batch_129k_hit_sweep(asd, dtype):
+    cfg = inputs.CONFIGS[3]
+    B, K, V = cfg["B"], cfg["K"], cfg["V"]
+    for pi, hit in enumerate(cfg["hits"]):
+        run_sequence(asd, B, K, V, dtype, range(3), cfg["gate"], cfg["cap"], cfg["budget"], 3,
+                     mix=inputs.mix_for_hit(hit), point=pi)
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+def test_ragged_shapes(asd, dtype):
+    rng = np.random.default_rng(5)
+    for V in (1, 2, 3, 7, 8, 9, 33, 1000, 1001, 4097, 70001):
+        for K in (0, 1, 5, 31):
+            for B in (1, 3):
+                b = inputs.gen_block(B, K, V, dtype, 10_000 + V * 64 + K * 4 + B, "cuda")
+                budget = float(rng.choice([0.0, 0.5, 4.0, math.inf]))
+                led = asd.make_ledger(B, budget)
+                g = gpu_verify(asd, b.logits, b.draft, led, 1.0, 2)
+                o = oracle.verify(b.logits.cpu(), b.draft.cpu().numpy(), np.array([[budget, 0.0]] * B, np.float32),
+                                  1.0, 2)
+                assert_parity(g, o, f"B={B} K={K} V={V}")
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+def test_misaligned_logits(asd, dtype):
+    B, K, V = 3, 4, 1003
+    for offset in range(1, 9):
+        flat = torch.empty(B * (K + 1) * V + offset, dtype=dtype, device="cuda")
+        b = inputs.gen_block(B, K, V, dtype, 777 + offset, "cuda")
+        view = flat[offset:].view(B, K + 1, V)
+        view.copy_(b.logits)
+        led = asd.make_ledger(B, 4.0)
+        g = gpu_verify(asd, view, b.draft, led, 1.0, 2)
+        o = oracle.verify(view.cpu(), b.draft.cpu().numpy(), np.array([[4.0, 0.0]] * B, np.float32), 1.0, 2)
+        assert_parity(g, o, f"offset {offset}")
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+def test_ties_zeros_and_infinities(asd, dtype):
+    rng = np.random.default_rng(6)
+    palette = np.array([-np.inf, -2.0, -0.0, 0.0, 1.5], np.float32)
+    B, K = 6, 7
+    for V in (5, 64, 999, 20000):
+        z = rng.choice(palette, size=(B, K + 1, V)).astype(np.float32)
+        z[0, :, :] = -np.inf                 # whole request at -inf: y* = 0 everywhere
+        z[1, :, :] = -0.0
+        z[1, :, V // 2:] = 0.0               # zeros of both signs: the first index wins
+        z[2, :, :] = 1.5                     # all equal
+        x = rng.integers(0, V, size=(B, K)).astype(np.int32)
+        x[3, :] = 0
+        t = torch.from_numpy(z).to(dtype).cuda()
+        xt = torch.from_numpy(x).cuda()
+        for budget in (0.0, 3.0):
+            led = asd.make_ledger(B, budget)
+            g = gpu_verify(asd, t, xt, led, math.inf, INT32_MAX)
+            o = oracle.verify(t.cpu(), x, np.array([[budget, 0.0]] * B, np.float32), math.inf, INT32_MAX)
+            assert_parity(g, o, f"V={V} budget={budget}")
+
+
+def test_status_flags(asd):
+    B, K, V = 6, 5, 3000
+    b = inputs.gen_block(B, K, V, torch.bfloat16, 99, "cuda")
+    logits, draft = b.logits.clone(), b.draft.clone()
+    draft[1, 3] = V            # out of range
+    draft[2, 0] = -4           # out of range
+    logits[3, 2, 1234] = float("nan")
+    led = asd.make_ledger(B, 4.0)
+    led[4] = torch.tensor([1.0, 2.0])          # spent > budget
+    led[5] = torch.tensor([float("nan"), 0.0])
+    led_before = led.cpu().numpy()
+    g = gpu_verify(asd, logits, draft, led, 1.0, 2)
+    o = oracle.verify(logits.cpu(), draft.cpu().numpy(), led_before, 1.0, 2)
+    assert list(g["status"]) == [0, 1, 1, 2, 4, 4]
+    assert_parity(g, o, "flags")
+    assert np.array_equal(g["ledger"][1:].view(np.uint32), led_before[1:].view(np.uint32))
+
+
+def test_infinite_controls_and_exhausted_ledger(asd):
+    B, K, V = 16, 8, 5000
+    b = inputs.gen_block(B, K, V, torch.float32, 4321, "cuda")
+    for (gate, cap, budget, spent) in ((math.inf, INT32_MAX, math.inf, 0.0), (0.0, 2, 4.0, 4.0),
+                                       (1.0, 0, 8.0, 0.0), (math.inf, INT32_MAX, 1e-30, 0.0)):
+        led = asd.make_ledger(B, budget, spent)
+        g = gpu_verify(asd, b.logits, b.draft, led, gate, cap)
+        o = oracle.verify(b.logits.cpu(), b.draft.cpu().numpy(), np.array([[budget, spent]] * B, np.float32),
+                          gate, cap)
+        assert_parity(g, o, f"controls {(gate, cap, budget, spent)}")
+
+
+def test_many_small_requests(asd):
+    """Many short rows per warp: each warp finishes and selects several requests."""
+    for (B, K, V) in ((3000, 31, 40), (5000, 3, 7), (700, 16, 130)):
+        b = inputs.gen_block(B, K, V, torch.bfloat16, B + K + V, "cuda")
+        led = asd.make_ledger(B, 2.0)
+        g = gpu_verify(asd, b.logits, b.draft, led, 0.5, 3)
+        o = oracle.verify(b.logits.cpu(), b.draft.cpu().numpy(), np.array([[2.0, 0.0]] * B, np.float32), 0.5, 3)
+        assert_parity(g, o, f"B={B} K={K} V={V}")
+
+
+def test_empty_batch_is_a_noop(asd):
+    logits = torch.empty(0, 9, 100, device="cuda")
+    draft = torch.empty(0, 8, dtype=torch.int32, device="cuda")
+    led = asd.make_ledger(0, 1.0)
+    out = asd.verify(logits, draft, led, 1.0, 2)
+    torch.cuda.synchronize()
+    assert out["accepted_len"].numel() == 0
+
+
+def test_one_workspace_serves_many_shapes(asd):
+    """The workspace resets itself: one buffer reused across shapes and entry points."""
+    ws = asd.Workspace(64, 31, 1, asd.F32)
+    rng = np.random.default_rng(8)
+    for i in range(20):
+        B, K, V = int(rng.integers(1, 64)), int(rng.integers(0, 32)), int(rng.integers(1, 3000))
+        dtype = torch.bfloat16 if i % 2 else torch.float32
+        b = inputs.gen_block(B, K, V, dtype, 555 + i, "cuda")
+        led = asd.make_ledger(B, 3.0)
+        out = asd.verify(b.logits, b.draft, led, 1.0, 2, workspace=ws) if i % 3 else \
+            asd.verify_strict(b.logits, b.draft, workspace=ws)
+        torch.cuda.synchronize()
+        g = _np(out)
+        g["ledger"] = led.cpu().numpy()
+        o = oracle.verify(b.logits.cpu(), b.draft.cpu().numpy(), np.array([[3.0, 0.0]] * B, np.float32), 1.0, 2,
+                          strict=(i % 3 == 0))
+        assert_parity(g, o, f"call {i}", ledger=bool(i % 3))
+
+
+def test_full_size_graph_launch_matches_oracle(asd):
+    """Qwen3-14B-shaped step (B=32, K=8, V=151936 bf16) in the benchmark's launch configuration:
+    rotating buffers larger than L2, steps captured in one CUDA graph, ledger carried."""
+    from paper_2608_03447_gb300.workload import VerifyWorkload
+    cfg = inputs.CONFIGS[1]
+    wl = VerifyWorkload(cfg["B"], cfg["K"], cfg["V"], cfg["dtype"], cfg["gate"], cfg["cap"], cfg["budget"],
+                        config=1, with_rows=True)
+    nsteps = 2 * wl.nbuf
+    graph = wl.capture(nsteps)
+    wl.reset_ledger()
+    graph.replay()
+    torch.cuda.synchronize()
+    led = np.array([[cfg["budget"], 0.0]] * cfg["B"], np.float32)
+    host = [(wl.logits[k].cpu(), wl.drafts[k].cpu().numpy()) for k in range(wl.nbuf)]
+    for i in range(nsteps):
+        z, x = host[i % wl.nbuf]
+        o = oracle.verify(z, x, led, cfg["gate"], cfg["cap"])
+        led = o["ledger"]
+    g = _np(wl.out)
+    g["ledger"] = wl.ledger.cpu().numpy()
+    assert_parity(g, o, "graph replay, last step")
