@@ -59,7 +59,8 @@ enum {
   ASD_ERR_WORKSPACE = 5, /* workspace smaller than the size query returns */
   ASD_ERR_ALIGN = 6,     /* pointer not aligned as documented */
   ASD_ERR_CUDA = 7,      /* a CUDA call failed (launch or device query) */
-  ASD_ERR_DEVICE = 8     /* the current device cannot run the kernel (not sm_103) */
+  ASD_ERR_DEVICE = 8,    /* the current device cannot run the kernel (not sm_103) */
+  ASD_ERR_TIMEOUT = 9    /* reported by asd_workspace_error: a kernel gave up waiting */
 };
 
 /* Per-request status bits (status[b]). */
@@ -77,9 +78,16 @@ int asd_workspace_size(int B, int K, int V, int dtype, size_t* bytes);
 
 /* Zero a workspace (cudaMemsetAsync on `stream`). Required once before the
  * first call that uses it; every verify call leaves the workspace zeroed again
- * when it completes, so it can be reused (and captured in a CUDA graph) with
- * no further initialisation. */
+ * when it completes, so it can be reused for any shape (and captured in a CUDA
+ * graph) with no further initialisation. */
 int asd_workspace_init(void* workspace, size_t bytes, asd_stream_t stream);
+
+/* Read the workspace's sticky error word (synchronises `stream`): 0, or
+ * ASD_ERR_TIMEOUT if a kernel that used this workspace gave up waiting on its
+ * own copy pipeline (a bounded wait of about one second; it does not happen in
+ * normal operation). After a non-zero word the outputs of that call are
+ * incomplete and the workspace must be re-initialised with asd_workspace_init. */
+int asd_workspace_error(const void* workspace, int* error, asd_stream_t stream);
 
 /*
  * ASD verification of B draft blocks (Eq. 1, 3, 5-13; Alg. 1).

@@ -49,6 +49,8 @@ def _declare(lib: ctypes.CDLL) -> ctypes.CDLL:
     lib.asd_workspace_size.restype = i32
     lib.asd_workspace_init.argtypes = [vp, sz, vp]
     lib.asd_workspace_init.restype = i32
+    lib.asd_workspace_error.argtypes = [vp, ctypes.POINTER(i32), vp]
+    lib.asd_workspace_error.restype = i32
     lib.asd_verify.argtypes = [vp, i32, i32, i32, i32, vp, vp, f32, i32, vp, vp, vp, vp, vp, vp, vp, sz, vp]
     lib.asd_verify.restype = i32
     lib.asd_verify_strict.argtypes = [vp, i32, i32, i32, i32, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
@@ -130,6 +132,12 @@ class Workspace:
     @property
     def ptr(self) -> int:
         return self.buffer.data_ptr()
+
+    def error(self, stream=None) -> int:
+        """The sticky error word (asd_workspace_error); synchronises the stream."""
+        word = ctypes.c_int(0)
+        _check("asd_workspace_error", load().asd_workspace_error(self.ptr, ctypes.byref(word), _stream(stream)))
+        return word.value
 
 
 def make_ledger(B: int, budget: float, spent: float = 0.0, device="cuda") -> torch.Tensor:

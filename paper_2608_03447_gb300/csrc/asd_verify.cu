@@ -23,16 +23,30 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <cstdlib>
 #include <mutex>
 
 #include "asd.h"
 
 namespace {
 
-constexpr int kThreads = 256;
+// Tuning constants (overridable at build time for launch-shape sweeps).
+#ifndef ASD_VERIFY_THREADS
+#define ASD_VERIFY_THREADS 256
+#endif
+#ifndef ASD_VERIFY_UNROLL
+#define ASD_VERIFY_UNROLL 4
+#endif
+#ifndef ASD_VERIFY_MIN_BLOCKS
+#define ASD_VERIFY_MIN_BLOCKS 0  // 0: no residency hint to the register allocator
+#endif
+#ifndef ASD_VERIFY_MIN_ELEMS_PER_WARP
+#define ASD_VERIFY_MIN_ELEMS_PER_WARP 2048
+#endif
+constexpr int kThreads = ASD_VERIFY_THREADS;
 constexpr int kWarpsPerBlock = kThreads / 32;
-constexpr int kUnroll = 4;                  // 128-bit loads in flight per lane
-constexpr long long kMinElemsPerWarp = 2048;
+constexpr int kUnroll = ASD_VERIFY_UNROLL;  // 128-bit loads in flight per lane
+constexpr long long kMinElemsPerWarp = ASD_VERIFY_MIN_ELEMS_PER_WARP;
 constexpr unsigned kFull = 0xffffffffu;
 
 struct VerifyParams {
@@ -55,6 +69,7 @@ struct VerifyParams {
   float* draft_logit;           // [B*(K+1)] z_j(x_j), written by the segment holding x_j
   unsigned long long* done;     // [B] elements finished, zero between calls
   unsigned int* flags;          // [B] ASD_STATUS_NAN_LOGIT bits, zero between calls
+  unsigned int* error;          // sticky: ASD_ERR_TIMEOUT when a pipeline wait gave up
 };
 
 // ---------------------------------------------------------------- element access
@@ -339,8 +354,14 @@ __device__ void select_request(const VerifyParams& p, int b, int lane) {
 
 // ---------------------------------------------------------------- the fused kernel
 
+#if ASD_VERIFY_MIN_BLOCKS > 0
+#define ASD_VERIFY_BOUNDS __launch_bounds__(kThreads, ASD_VERIFY_MIN_BLOCKS)
+#else
+#define ASD_VERIFY_BOUNDS __launch_bounds__(kThreads)
+#endif
+
 template <typename T, bool kStrict>
-__global__ void __launch_bounds__(kThreads) verify_kernel(const VerifyParams p) {
+__global__ void ASD_VERIFY_BOUNDS verify_kernel(const VerifyParams p) {
   const int lane = threadIdx.x & 31;
   const long long warp = static_cast<long long>(blockIdx.x) * kWarpsPerBlock + (threadIdx.x >> 5);
   const long long lo = warp == 0 ? 0 : p.head + warp * p.per_warp;
@@ -403,23 +424,568 @@ __global__ void __launch_bounds__(kThreads) verify_kernel(const VerifyParams p) 
   }
 }
 
+// ---------------------------------------------------------------- TMA pipeline kernel
+//
+// One CTA per SM. The CTA owns an equal, 16-byte aligned slice of the flat
+// logits and streams it through a ring of shared-memory stages with bulk
+// copies (cp.async.bulk, completion counted on an mbarrier). A producer warp
+// keeps every free stage in flight, so the bytes in flight per SM are set by
+// the ring (kTmaStages x kTmaChunkBytes), not by registers. The consumer warps
+// each take a fixed sub-range of every chunk, so a warp visits its elements in
+// increasing order and keeps one running (value, index) per lane for the row
+// it is in; it flushes the row's key when it crosses into the next row, and
+// adds its element count to the request's counter when it crosses into the
+// next request (the last one to finish a request runs its selection).
+// Every wait is bounded (about a second of %globaltimer); on a timeout the CTA
+// records ASD_ERR_TIMEOUT in the workspace, stops, and drains its own copies.
+
+#ifndef ASD_TMA_STAGES
+#define ASD_TMA_STAGES 6  // 6 x 16 KB: two CTAs (this launch and the next) fit on one SM
+#endif
+#ifndef ASD_TMA_CHUNK_BYTES
+#define ASD_TMA_CHUNK_BYTES 16384
+#endif
+#ifndef ASD_TMA_CONSUMER_WARPS
+#define ASD_TMA_CONSUMER_WARPS 8
+#endif
+#ifndef ASD_TMA_POLL
+#define ASD_TMA_POLL 0  // 0: mbarrier.try_wait (may suspend), 1: mbarrier.test_wait spin
+#endif
+#ifndef ASD_TMA_L2_HINT
+#define ASD_TMA_L2_HINT 1  // evict-first L2 policy on the streamed logits
+#endif
+constexpr int kTmaStages = ASD_TMA_STAGES;
+constexpr int kTmaChunkBytes = ASD_TMA_CHUNK_BYTES;
+constexpr int kTmaConsumers = ASD_TMA_CONSUMER_WARPS;
+constexpr int kTmaThreads = (kTmaConsumers + 1) * 32;
+constexpr unsigned long long kWaitLimitNs = 1000000000ull;
+static_assert(kTmaChunkBytes % (16 * 32 * kTmaConsumers) == 0,
+              "every consumer warp takes whole 128-bit vectors of each chunk, one per lane per pass");
+
+// Rows of one CTA's slice merged in shared memory until the end of the stream
+// (then flushed to the workspace once); slices spanning more rows than this
+// merge straight into the workspace.
+constexpr int kRowTable = 256;
+
+struct TmaShared {
+  uint4 ring[kTmaStages][kTmaChunkBytes / 16];
+  unsigned long long full[kTmaStages];
+  unsigned long long empty[kTmaStages];
+  unsigned long long row_key[kRowTable];  // merged (value, index) keys of the slice's rows
+  float row_zx[kRowTable];                // the draft token's logit of each row, if seen here
+  unsigned int row_bits[kRowTable];       // 1: a NaN was seen, 2: row_zx is valid
+  int abort;
+};
+
+__device__ __forceinline__ uint32_t smem_u32(const void* ptr) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(ptr));
+}
+__device__ __forceinline__ void mbar_init(unsigned long long* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(unsigned long long* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(unsigned long long* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(unsigned long long* bar, uint32_t parity) {
+  uint32_t done;
+#if ASD_TMA_POLL
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(done)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+#else
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(done)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+#endif
+  return done != 0;
+}
+__device__ __forceinline__ unsigned long long global_ns() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+// Waits for the phase with the given parity; false on timeout or when another
+// warp of the CTA has given up.
+__device__ bool mbar_wait(unsigned long long* bar, uint32_t parity, volatile int* abort) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const unsigned long long t0 = global_ns();
+  for (unsigned it = 1;; ++it) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((it & 255u) == 0) {  // the clock and the abort flag are checked now and then
+      if (*abort) return false;
+      if (global_ns() - t0 > kWaitLimitNs) return false;
+    }
+  }
+}
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes,
+                                          unsigned long long* bar, unsigned long long policy) {
+#if ASD_TMA_L2_HINT
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1], %2, [%3], %4;" ::"r"(smem_u32(dst)),
+      "l"(src), "r"(bytes), "r"(smem_u32(bar)), "l"(policy)
+      : "memory");
+#else
+  (void)policy;
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1], %2, [%3];" ::"r"(smem_u32(dst)),
+      "l"(src), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+#endif
+}
+__device__ __forceinline__ unsigned long long evict_first_policy() {
+  unsigned long long pol;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+__device__ __forceinline__ uint4 lds128(const uint4* p) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "r"(smem_u32(p)));
+  return v;
+}
+
+// Programmatic dependent launch: the next launch on the stream may start once
+// every CTA of this one has signalled; it waits for this launch to complete
+// (and its writes to be visible) before its first access to the workspace,
+// the ledger or the outputs. Its logits stream in the meantime.
+__device__ __forceinline__ void pdl_signal_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait_prerequisites() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
+// Element `off` of a staged chunk, read with ld.shared (src is a shared-memory
+// pointer: the global-only loads of Elem<T>::load must never see it).
+__device__ __forceinline__ float smem_elem(const uint4* src, int off, float) {
+  float v;
+  asm volatile("ld.shared.f32 %0, [%1];" : "=f"(v) : "r"(smem_u32(src) + 4u * static_cast<uint32_t>(off)));
+  return v;
+}
+__device__ __forceinline__ float smem_elem(const uint4* src, int off, __nv_bfloat16) {
+  unsigned short bits;
+  asm volatile("ld.shared.u16 %0, [%1];" : "=h"(bits) : "r"(smem_u32(src) + 2u * static_cast<uint32_t>(off)));
+  return __uint_as_float(static_cast<uint32_t>(bits) << 16);
+}
+
+// The first element of v equal to m, its maximum; VN - 1 if none (m is NaN).
+template <typename T>
+__device__ __forceinline__ int vec_first_equal(const uint4& v, float m) {
+  int first = Elem<T>::kVec - 1;
+#pragma unroll
+  for (int t = Elem<T>::kVec - 1; t >= 0; --t)
+    if (Elem<T>::lane(v, t) == m) first = t;
+  return first;
+}
+
+// A request's last counted elements: the warp that completes the request runs
+// its selection. Out of line: it runs a few times per launch.
+template <typename T, bool kStrict>
+__device__ __noinline__ void finish_request(const VerifyParams& p, int b, unsigned long long pend, int lane) {
+  const unsigned long long request_elems = static_cast<unsigned long long>(p.K + 1) * p.V;
+  bool last = false;
+  if (lane == 0) {
+    __threadfence();
+    const unsigned long long old = atomicAdd(&p.done[b], pend);
+    last = old + pend == request_elems;
+  }
+  if (__shfl_sync(kFull, last, 0)) {
+    __threadfence();
+    select_request<T, kStrict>(p, b, lane);
+  }
+}
+
+// Merges one warp's partial result for a row into the workspace: the row's
+// key, its NaN flag and (from the lane that holds it) the draft token's logit.
+// The first global write of a warp: it waits for the previous launch first.
+__device__ __noinline__ void flush_row_key(const VerifyParams& p, long long row, int b,
+                                           unsigned long long key, bool nan, bool has_zx, float zx,
+                                           int lane) {
+  pdl_wait_prerequisites();
+  key = warp_max_key(key);
+  nan = __any_sync(kFull, nan);
+  if (lane == 0) {
+    if (key) atomicMax(&p.row_key[row], key);
+    if (nan) atomicOr(&p.flags[b], ASD_STATUS_NAN_LOGIT);
+  }
+  if (has_zx) p.draft_logit[row] = zx;
+}
+
+// Per-warp cursor: the row and request the warp is in (warp-uniform) and each
+// lane's running candidate for that row. Offsets are relative to the row start.
+struct RowCursor {
+  long long row;            // current row
+  long long row0, row1;     // its flat element range [row0, row1)
+  int b;                    // its request
+  int x;                    // its draft id, -1 for the bonus row or an id outside [0, V)
+  int next_x;               // prefetched draft id of row + 1
+  float best;               // per lane: NaN-propagating maximum over whole vectors
+  int saved_rel;            // per lane: offset of the vector that first reached best, -1 none
+  uint4 saved;              // per lane: that vector
+  int first_rel;            // per lane: offset of the lane's first vector in the row, -1 none
+  float sbest;              // per lane: best single element seen at row boundaries
+  int sidx;                 // per lane: its offset, -1 none
+  bool snan;                // per lane: a single element was NaN
+  float zx;                 // per lane: the draft token's logit, if this lane saw it
+  bool has_zx;
+};
+
+__device__ __forceinline__ int draft_of_row(const VerifyParams& p, long long row) {
+  const int K1 = p.K + 1;
+  const long long b = row / K1;
+  const int j = static_cast<int>(row - b * K1);
+  if (j >= p.K || b >= p.B) return -1;
+  return __ldg(p.draft + b * p.K + j);
+}
+
+__device__ __forceinline__ void cursor_enter(RowCursor& c, const VerifyParams& p, long long row) {
+  c.row = row;
+  c.row0 = row * p.V;
+  c.row1 = c.row0 + p.V;
+  c.b = static_cast<int>(row / (p.K + 1));
+  c.x = (c.next_x >= 0 && c.next_x < p.V) ? c.next_x : -1;
+  c.next_x = draft_of_row(p, row + 1);  // consumed at the next row change
+  c.best = -INFINITY;
+  c.saved_rel = -1;
+  c.saved = make_uint4(0, 0, 0, 0);
+  c.first_rel = -1;
+  c.sbest = -INFINITY;
+  c.sidx = -1;
+  c.snan = false;
+  c.zx = 0.0f;
+  c.has_zx = false;
+}
+
+// Where a warp's finished rows go: the CTA's row table (rows table_row0 ..)
+// or, when the slice spans too many rows, the workspace directly.
+struct RowSink {
+  TmaShared* sh;
+  long long table_row0;
+  bool table;
+};
+
+template <typename T>
+__device__ __forceinline__ void cursor_flush_row(RowCursor& c, const VerifyParams& p, const RowSink& sink,
+                                                 int lane) {
+  float v = -INFINITY;
+  int idx = -1;
+  if (c.saved_rel >= 0) {
+    v = c.best;
+    idx = c.saved_rel + vec_first_equal<T>(c.saved, c.best);
+  } else if (c.first_rel >= 0) {
+    idx = c.first_rel;  // every whole-vector value this lane saw was -inf (or NaN, flagged)
+  }
+  if (c.sidx >= 0 && (idx < 0 || c.sbest > v || (c.sbest == v && c.sidx < idx))) {
+    v = c.sbest;
+    idx = c.sidx;
+  }
+  const unsigned long long key = idx < 0 ? 0ull : make_key(v, static_cast<uint32_t>(idx));
+  const bool nan = c.snan || c.best != c.best;
+  if (!sink.table) {
+    flush_row_key(p, c.row, c.b, key, nan, c.has_zx, c.zx, lane);
+    return;
+  }
+  const int t = static_cast<int>(c.row - sink.table_row0);
+  const unsigned long long wkey = warp_max_key(key);
+  const bool wnan = __any_sync(kFull, nan);
+  if (lane == 0) {
+    if (wkey) atomicMax(&sink.sh->row_key[t], wkey);
+    if (wnan) atomicOr(&sink.sh->row_bits[t], 1u);
+  }
+  if (c.has_zx) {
+    sink.sh->row_zx[t] = c.zx;
+    atomicOr(&sink.sh->row_bits[t], 2u);
+  }
+}
+
+// Moves the cursor to the row holding flat element e, flushing what it leaves.
+template <typename T>
+__device__ __forceinline__ void cursor_advance(RowCursor& c, const VerifyParams& p, const RowSink& sink,
+                                               long long e, int lane) {
+  cursor_flush_row<T>(c, p, sink, lane);
+  const long long row = e / p.V;
+  if (row != c.row + 1) c.next_x = draft_of_row(p, row);  // rows in between belong to other warps
+  cursor_enter(c, p, row);
+}
+
+// One element at row offset rel (row boundaries, ragged head and tail).
+__device__ __forceinline__ void lane_element(RowCursor& c, const VerifyParams& p, float v, int rel) {
+  if (v != v) {
+    c.snan = true;
+  } else if (c.sidx < 0 || v > c.sbest) {
+    c.sbest = v;
+    c.sidx = rel;
+  }
+  if (rel == c.x) {
+    c.zx = v;
+    c.has_zx = true;
+  }
+}
+
+// Elements [a, a + 32*VN*kPasses) of the flat array, staged at `src`, one
+// vector per lane per pass (vector u*32 + lane); elements at or past `limit`
+// are not data.
+template <typename T, bool kStrict, int kPasses>
+__device__ __forceinline__ void consume_span(RowCursor& c, const VerifyParams& p, const RowSink& sink,
+                                             const uint4* src, long long a, long long limit, int lane) {
+  constexpr int VN = Elem<T>::kVec;
+  constexpr int kSpan = kPasses * 32 * VN;
+  const long long span_end = a + kSpan;
+  if (span_end <= c.row1 && span_end <= limit) {
+    // fast path: the whole span lies in the current row; no branches per vector
+    uint4 v[kPasses];
+#pragma unroll
+    for (int u = 0; u < kPasses; ++u) v[u] = lds128(src + u * 32 + lane);
+    const int a_rel = static_cast<int>(a - c.row0);
+    if (c.first_rel < 0) c.first_rel = a_rel + lane * VN;
+#pragma unroll
+    for (int u = 0; u < kPasses; ++u) {
+      const float m = vec_max(v[u], T());
+      const bool gt = m > c.best;
+      c.best = fmax_nan(c.best, m);
+      c.saved.x = gt ? v[u].x : c.saved.x;
+      c.saved.y = gt ? v[u].y : c.saved.y;
+      c.saved.z = gt ? v[u].z : c.saved.z;
+      c.saved.w = gt ? v[u].w : c.saved.w;
+      c.saved_rel = gt ? a_rel + (u * 32 + lane) * VN : c.saved_rel;
+    }
+    const int off = c.x - a_rel;  // the draft token's logit, if this span holds it
+    if (static_cast<unsigned>(off) < static_cast<unsigned>(kSpan) && lane == 0) {
+      c.zx = smem_elem(src, off, T());
+      c.has_zx = true;
+    }
+    return;
+  }
+  // slow path: row boundaries (or the end of the data) inside the span
+  const long long end = span_end < limit ? span_end : limit;
+#pragma unroll 1
+  for (int u = 0; u < kPasses; ++u) {
+    const long long g0 = a + static_cast<long long>(u) * 32 * VN;  // this pass covers [g0, g0 + 32 VN)
+    if (g0 >= end) break;
+    const long long g1 = g0 + 32 * VN < end ? g0 + 32 * VN : end;
+    const long long e0 = g0 + static_cast<long long>(lane) * VN;    // this lane's vector
+    uint4 v = make_uint4(0, 0, 0, 0);
+    if (e0 < g1) v = lds128(src + u * 32 + lane);
+    long long pos = g0;
+    while (pos < g1) {  // warp-uniform: one row of the pass at a time
+      if (pos >= c.row1) cursor_advance<T>(c, p, sink, pos, lane);
+      const long long seg_end = g1 < c.row1 ? g1 : c.row1;
+#pragma unroll
+      for (int t = 0; t < VN; ++t) {
+        const long long e = e0 + t;
+        if (e >= pos && e < seg_end) lane_element(c, p, Elem<T>::lane(v, t), static_cast<int>(e - c.row0));
+      }
+      pos = seg_end;
+    }
+  }
+}
+
+// Single elements [from, to) read from global memory (the ragged head and tail).
+template <typename T, bool kStrict>
+__device__ __forceinline__ void consume_loose(RowCursor& c, const VerifyParams& p, const RowSink& sink,
+                                              long long from, long long to, int lane) {
+  const T* z = static_cast<const T*>(p.logits);
+  for (long long pos = from; pos < to;) {
+    if (pos >= c.row1) cursor_advance<T>(c, p, sink, pos, lane);
+    const long long seg_end = to < c.row1 ? to : c.row1;
+    const long long e = pos + lane;
+    if (e < seg_end) lane_element(c, p, Elem<T>::load(z, e), static_cast<int>(e - c.row0));
+    pos = seg_end;
+  }
+}
+
+template <typename T, bool kStrict>
+__global__ void __launch_bounds__(kTmaThreads, 1)
+    verify_tma_kernel(const __grid_constant__ VerifyParams p, long long bulk_end, long long per_cta) {
+  constexpr int VN = Elem<T>::kVec;
+  constexpr int kChunkElems = kTmaChunkBytes / static_cast<int>(sizeof(T));
+  constexpr int kWarpElems = kChunkElems / kTmaConsumers;  // one consumer's share of a chunk
+  constexpr int kPasses = kWarpElems / (32 * VN);          // vectors per lane per chunk
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  TmaShared& sh = *reinterpret_cast<TmaShared*>(smem_raw);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const T* z = static_cast<const T*>(p.logits);
+
+  // this CTA's slice [lo, hi) of the bulk region [p.head, bulk_end)
+  const long long lo = p.head + static_cast<long long>(blockIdx.x) * per_cta;
+  long long hi = lo + per_cta;
+  hi = hi < bulk_end ? hi : bulk_end;
+  const int nchunks = lo < hi ? static_cast<int>((hi - lo + kChunkElems - 1) / kChunkElems) : 0;
+
+  pdl_signal_dependents();
+
+  // each consumer's first row is known now: start its draft-id load before the
+  // first copy lands
+  RowCursor c;
+  c.next_x = -1;
+  const long long first_a = lo + static_cast<long long>(warp) * kWarpElems;
+  const bool head_here = blockIdx.x == 0 && warp == 0 && p.head > 0;
+  if (warp < kTmaConsumers) c.next_x = draft_of_row(p, head_here ? 0 : (first_a < hi ? first_a : 0) / p.V);
+
+  // this CTA's rows, including the ragged head (CTA 0) and tail (last CTA)
+  const long long cta_lo = blockIdx.x == 0 ? 0 : lo;
+  const long long cta_hi = blockIdx.x == gridDim.x - 1 ? p.total : hi;
+  RowSink sink;
+  sink.sh = &sh;
+  sink.table_row0 = cta_lo / p.V;
+  const long long table_rows = cta_lo < cta_hi ? (cta_hi - 1) / p.V - sink.table_row0 + 1 : 0;
+  sink.table = table_rows <= kRowTable;
+  for (int t = threadIdx.x; t < kRowTable; t += blockDim.x) {
+    sh.row_key[t] = 0ull;
+    sh.row_bits[t] = 0u;
+  }
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kTmaStages; ++s) {
+      mbar_init(&sh.full[s], 1);
+      mbar_init(&sh.empty[s], kTmaConsumers);
+    }
+    sh.abort = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  __syncthreads();
+
+  int issued = 0;  // producer: chunks issued
+  if (warp == kTmaConsumers) {
+    if (lane == 0) {
+      const unsigned long long policy = evict_first_policy();
+      for (int ch = 0; ch < nchunks; ++ch) {
+        const int s = ch % kTmaStages;
+        if (ch >= kTmaStages && !mbar_wait(&sh.empty[s], ((ch / kTmaStages) - 1) & 1, &sh.abort)) {
+          sh.abort = 1;
+          atomicExch(p.error, static_cast<unsigned>(ASD_ERR_TIMEOUT));
+          break;
+        }
+        const long long e0 = lo + static_cast<long long>(ch) * kChunkElems;
+        const long long n = hi - e0 < kChunkElems ? hi - e0 : kChunkElems;
+        const uint32_t bytes = static_cast<uint32_t>(n * sizeof(T));
+        mbar_expect_tx(&sh.full[s], bytes);
+        bulk_load(sh.ring[s], z + e0, bytes, &sh.full[s], policy);
+        issued = ch + 1;
+      }
+    }
+  } else {
+    bool started = false;
+
+    // the ragged head [0, p.head) (fewer than VN elements) belongs to CTA 0, warp 0
+    if (head_here) {
+      cursor_enter(c, p, 0);
+      started = true;
+      consume_loose<T, kStrict>(c, p, sink, 0, p.head, lane);
+    }
+
+    for (int ch = 0; ch < nchunks; ++ch) {
+      const int s = ch % kTmaStages;
+      // every lane observes the phase itself (that makes the staged bytes visible
+      // to it); the warp proceeds only if all lanes did
+      const bool ok = __all_sync(kFull, mbar_wait(&sh.full[s], (ch / kTmaStages) & 1, &sh.abort));
+      if (!ok) {
+        sh.abort = 1;
+        if (lane == 0) atomicExch(p.error, static_cast<unsigned>(ASD_ERR_TIMEOUT));
+        break;
+      }
+      const long long a = lo + static_cast<long long>(ch) * kChunkElems + static_cast<long long>(warp) * kWarpElems;
+      if (a < hi) {
+        if (!started) {
+          cursor_enter(c, p, a / p.V);  // its draft id was loaded at kernel start
+          started = true;
+        } else if (a >= c.row1) {
+          cursor_advance<T>(c, p, sink, a, lane);
+        }
+        consume_span<T, kStrict, kPasses>(c, p, sink, sh.ring[s] + warp * (kWarpElems / VN), a, hi, lane);
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sh.empty[s]);
+    }
+
+    // the ragged tail [bulk_end, total) (fewer than VN elements): last CTA, last consumer
+    if (!sh.abort && blockIdx.x == gridDim.x - 1 && warp == kTmaConsumers - 1 && bulk_end < p.total) {
+      if (!started) {
+        c.next_x = draft_of_row(p, bulk_end / p.V);
+        cursor_enter(c, p, bulk_end / p.V);
+        started = true;
+      }
+      consume_loose<T, kStrict>(c, p, sink, bulk_end, p.total, lane);
+    }
+    if (started && !sh.abort) cursor_flush_row<T>(c, p, sink, lane);
+    __threadfence();  // this warp's key merges and draft-logit stores, before the counts below
+  }
+
+  __syncthreads();
+  if (sh.abort) {
+    // after a timeout: wait (bounded) for this CTA's copies still in flight, then leave
+    if (warp == kTmaConsumers && lane == 0) {
+      for (int ch = issued > kTmaStages ? issued - kTmaStages : 0; ch < issued; ++ch) {
+        const int s = ch % kTmaStages;
+        const unsigned long long t0 = global_ns();
+        while (!mbar_try_wait(&sh.full[s], (ch / kTmaStages) & 1) && global_ns() - t0 < kWaitLimitNs) {
+        }
+      }
+    }
+    return;
+  }
+  // The first touch of the workspace: wait for the previous launch, flush the
+  // row table, then count this CTA's elements of each request it touched; the
+  // CTA that completes a request runs its selection.
+  pdl_wait_prerequisites();
+  if (sink.table) {
+    for (int t = threadIdx.x; t < table_rows; t += blockDim.x) {
+      const long long row = sink.table_row0 + t;
+      const unsigned long long key = sh.row_key[t];
+      const unsigned bits = sh.row_bits[t];
+      if (key) atomicMax(&p.row_key[row], key);
+      if (bits & 1u) atomicOr(&p.flags[row / (p.K + 1)], ASD_STATUS_NAN_LOGIT);
+      if (bits & 2u) p.draft_logit[row] = sh.row_zx[t];
+    }
+    __threadfence();
+    __syncthreads();
+  }
+  if (cta_lo < cta_hi) {
+    const long long rv = static_cast<long long>(p.K + 1) * p.V;
+    const long long b_first = cta_lo / rv, b_last = (cta_hi - 1) / rv;
+    for (long long b = b_first + warp; b <= b_last; b += kTmaConsumers + 1) {
+      const long long r0 = b * rv > cta_lo ? b * rv : cta_lo;
+      const long long r1 = (b + 1) * rv < cta_hi ? (b + 1) * rv : cta_hi;
+      finish_request<T, kStrict>(p, static_cast<int>(b), static_cast<unsigned long long>(r1 - r0), lane);
+    }
+  }
+}
+
 // ---------------------------------------------------------------- host side
 
 inline size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
+// Workspace: the error word first (fixed offset for asd_workspace_error), then
+// the per-row and per-request slots.
 struct WorkspaceLayout {
-  size_t row_key, draft_logit, done, flags, total;
+  size_t error, row_key, draft_logit, done, flags, total;
 };
 
 WorkspaceLayout layout_for(int B, int K) {
   const size_t R = static_cast<size_t>(B) * (K + 1);
   WorkspaceLayout l;
-  l.row_key = 0;
+  l.error = 0;
+  l.row_key = 256;
   l.draft_logit = align_up(l.row_key + 8 * R, 256);
   l.done = align_up(l.draft_logit + 4 * R, 256);
   l.flags = align_up(l.done + 8 * static_cast<size_t>(B), 256);
   l.total = align_up(l.flags + 4 * static_cast<size_t>(B), 256);
-  if (l.total == 0) l.total = 256;
   return l;
 }
 
@@ -459,8 +1025,95 @@ int resident_warps(int* out) {
   return ASD_OK;
 }
 
+struct DeviceInfo {
+  int sms = 0;
+  bool tma_ready[4] = {false, false, false, false};
+};
+
+// SM count of the current device, and the one-time dynamic shared memory
+// opt-in of the TMA kernels, cached per device.
+int device_info(int* dev_out, DeviceInfo** info_out) {
+  constexpr int kMaxDevices = 64;
+  static DeviceInfo info[kMaxDevices];
+  static std::mutex mu;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return ASD_ERR_CUDA;
+  if (dev < 0 || dev >= kMaxDevices) return ASD_ERR_DEVICE;
+  std::lock_guard<std::mutex> g(mu);
+  if (info[dev].sms == 0) {
+    int sms = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return ASD_ERR_CUDA;
+    info[dev].sms = sms;
+  }
+  *dev_out = dev;
+  *info_out = &info[dev];
+  return ASD_OK;
+}
+
+template <typename T, bool kStrict>
+int launch_tma(VerifyParams& p, cudaStream_t stream) {
+  constexpr int VN = Elem<T>::kVec;
+  constexpr long long kMinPerCta = 2LL * kTmaChunkBytes / static_cast<long long>(sizeof(T));
+  const uintptr_t addr = reinterpret_cast<uintptr_t>(p.logits);
+  if (addr % sizeof(T) != 0) return ASD_ERR_ALIGN;
+  long long head = static_cast<long long>(((16 - addr % 16) % 16) / sizeof(T));
+  if (head > p.total) head = p.total;
+  const long long bulk = (p.total - head) / VN * VN;
+  int dev = 0;
+  DeviceInfo* info = nullptr;
+  int rc = device_info(&dev, &info);
+  if (rc != ASD_OK) return rc;
+  const int slot = (sizeof(T) == 2 ? 2 : 0) + (kStrict ? 1 : 0);
+  if (!info->tma_ready[slot]) {
+    if (cudaFuncSetAttribute(verify_tma_kernel<T, kStrict>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(sizeof(TmaShared))) != cudaSuccess)
+      return ASD_ERR_CUDA;
+    info->tma_ready[slot] = true;
+  }
+  long long ncta = (bulk + kMinPerCta - 1) / kMinPerCta;
+  if (ncta > info->sms) ncta = info->sms;
+  if (ncta < 1) ncta = 1;
+  long long per_cta = (bulk + ncta - 1) / ncta;
+  per_cta = (per_cta + VN - 1) / VN * VN;
+  if (per_cta < VN) per_cta = VN;
+  ncta = bulk > 0 ? (bulk + per_cta - 1) / per_cta : 1;
+  p.head = head;
+  p.per_warp = 0;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(ncta));
+  cfg.blockDim = dim3(kTmaThreads);
+  cfg.dynamicSmemBytes = sizeof(TmaShared);
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  const char* env = getenv("ASD_VERIFY_PDL");
+  if (!(env && env[0] == '0')) {
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+  }
+  const long long bulk_end = head + bulk;
+  if (cudaLaunchKernelEx(&cfg, verify_tma_kernel<T, kStrict>, p, bulk_end, per_cta) != cudaSuccess)
+    return ASD_ERR_CUDA;
+  return cudaGetLastError() == cudaSuccess ? ASD_OK : ASD_ERR_CUDA;
+}
+
+// Which kernel streams the logits: the TMA pipeline for inputs of at least
+// kTmaMinBytes, the register-streaming kernel below that (fewer, shorter
+// warps start faster on tiny inputs). ASD_VERIFY_KERNEL=stream|tma in the
+// environment overrides the choice (used by the tests to cover both kernels).
+constexpr long long kTmaMinBytes = 1LL << 20;
+
+bool use_tma(long long bytes) {
+  const char* env = getenv("ASD_VERIFY_KERNEL");
+  if (env && env[0] == 't') return true;
+  if (env && env[0] == 's') return false;
+  return bytes >= kTmaMinBytes;
+}
+
 template <typename T, bool kStrict>
 int launch(VerifyParams& p, cudaStream_t stream) {
+  if (use_tma(p.total * static_cast<long long>(sizeof(T)))) return launch_tma<T, kStrict>(p, stream);
   constexpr int VN = Elem<T>::kVec;
   const uintptr_t addr = reinterpret_cast<uintptr_t>(p.logits);
   if (addr % sizeof(T) != 0) return ASD_ERR_ALIGN;
@@ -526,6 +1179,7 @@ int verify_common(bool strict, const void* logits, int dtype, int B, int K, int 
   p.draft_logit = reinterpret_cast<float*>(ws + l.draft_logit);
   p.done = reinterpret_cast<unsigned long long*>(ws + l.done);
   p.flags = reinterpret_cast<unsigned int*>(ws + l.flags);
+  p.error = reinterpret_cast<unsigned int*>(ws + l.error);
 
   if (dtype == ASD_F32)
     return strict ? launch<float, true>(p, stream) : launch<float, false>(p, stream);
@@ -541,6 +1195,17 @@ int asd_workspace_size(int B, int K, int V, int dtype, size_t* bytes) {
   const int rc = check_shape(B, K, V, dtype);
   if (rc != ASD_OK) return rc;
   *bytes = layout_for(B, K).total;
+  return ASD_OK;
+}
+
+int asd_workspace_error(const void* workspace, int* error, asd_stream_t stream) {
+  if (!workspace || !error) return ASD_ERR_NULL;
+  unsigned int word = 0;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (cudaMemcpyAsync(&word, workspace, sizeof word, cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess)
+    return ASD_ERR_CUDA;
+  *error = static_cast<int>(word);
   return ASD_OK;
 }
 
@@ -580,6 +1245,7 @@ const char* asd_status_string(int code) {
     case ASD_ERR_ALIGN: return "pointer misaligned";
     case ASD_ERR_CUDA: return "CUDA call failed";
     case ASD_ERR_DEVICE: return "the current device cannot run this kernel";
+    case ASD_ERR_TIMEOUT: return "a kernel gave up waiting on its own pipeline (outputs incomplete)";
     default: return "unknown status code";
   }
 }

@@ -19,6 +19,13 @@ pytestmark = pytest.mark.gpu
 INT32_MAX = 2**31 - 1
 
 
+@pytest.fixture(params=["stream", "tma"])
+def kernel(request, monkeypatch):
+    """Runs the test through the register-streaming kernel and through the TMA pipeline kernel."""
+    monkeypatch.setenv("ASD_VERIFY_KERNEL", request.param)
+    return request.param
+
+
 def _np(out: dict) -> dict:
     return {k: v.cpu().numpy() for k, v in out.items()}
 
@@ -71,14 +78,14 @@ def run_sequence(asd, B, K, V, dtype, blocks, gate, cap, budget, config, mix=inp
     return led_orc
 
 
-def test_tiny_fp32_sixteen_blocks(asd):
+def test_tiny_fp32_sixteen_blocks(asd, kernel):
     cfg = inputs.CONFIGS[0]
     led = run_sequence(asd, cfg["B"], cfg["K"], cfg["V"], cfg["dtype"], range(cfg["blocks"]),
                        cfg["gate"], cfg["cap"], cfg["budget"], 0)
     assert np.all(led[:, 1] <= cfg["budget"])
 
 
-def test_tiny_zero_budget_is_strict(asd):
+def test_tiny_zero_budget_is_strict(asd, kernel):
     cfg = inputs.CONFIGS[0]
     B, K, V = cfg["B"], cfg["K"], cfg["V"]
     for blk in range(cfg["blocks"]):
@@ -91,7 +98,7 @@ def test_tiny_zero_budget_is_strict(asd):
         assert np.array_equal(g["ledger"], np.zeros((B, 2), np.float32))
 
 
-def test_qwen3_shape_bf16_blocks(asd):
+def test_qwen3_shape_bf16_blocks(asd, kernel):
     cfg = inputs.CONFIGS[1]
     run_sequence(asd, cfg["B"], cfg["K"], cfg["V"], cfg["dtype"], range(8), cfg["gate"], cfg["cap"],
                  cfg["budget"], 1)
@@ -134,7 +141,7 @@ def test_large_batch_129k_hit_sweep(asd, dtype):
 
 
 @pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
-def test_ragged_shapes(asd, dtype):
+def test_ragged_shapes(asd, kernel, dtype):
     rng = np.random.default_rng(5)
     for V in (1, 2, 3, 7, 8, 9, 33, 1000, 1001, 4097, 70001):
         for K in (0, 1, 5, 31):
@@ -149,7 +156,7 @@ def test_ragged_shapes(asd, dtype):
 
 
 @pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
-def test_misaligned_logits(asd, dtype):
+def test_misaligned_logits(asd, kernel, dtype):
     B, K, V = 3, 4, 1003
     for offset in range(1, 9):
         flat = torch.empty(B * (K + 1) * V + offset, dtype=dtype, device="cuda")
@@ -163,7 +170,7 @@ def test_misaligned_logits(asd, dtype):
 
 
 @pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
-def test_ties_zeros_and_infinities(asd, dtype):
+def test_ties_zeros_and_infinities(asd, kernel, dtype):
     rng = np.random.default_rng(6)
     palette = np.array([-np.inf, -2.0, -0.0, 0.0, 1.5], np.float32)
     B, K = 6, 7
@@ -184,7 +191,7 @@ def test_ties_zeros_and_infinities(asd, dtype):
             assert_parity(g, o, f"V={V} budget={budget}")
 
 
-def test_status_flags(asd):
+def test_status_flags(asd, kernel):
     B, K, V = 6, 5, 3000
     b = inputs.gen_block(B, K, V, torch.bfloat16, 99, "cuda")
     logits, draft = b.logits.clone(), b.draft.clone()
@@ -202,7 +209,7 @@ def test_status_flags(asd):
     assert np.array_equal(g["ledger"][1:].view(np.uint32), led_before[1:].view(np.uint32))
 
 
-def test_infinite_controls_and_exhausted_ledger(asd):
+def test_infinite_controls_and_exhausted_ledger(asd, kernel):
     B, K, V = 16, 8, 5000
     b = inputs.gen_block(B, K, V, torch.float32, 4321, "cuda")
     for (gate, cap, budget, spent) in ((math.inf, INT32_MAX, math.inf, 0.0), (0.0, 2, 4.0, 4.0),
@@ -214,7 +221,7 @@ def test_infinite_controls_and_exhausted_ledger(asd):
         assert_parity(g, o, f"controls {(gate, cap, budget, spent)}")
 
 
-def test_many_small_requests(asd):
+def test_many_small_requests(asd, kernel):
     """Many short rows per warp: each warp finishes and selects several requests."""
     for (B, K, V) in ((3000, 31, 40), (5000, 3, 7), (700, 16, 130)):
         b = inputs.gen_block(B, K, V, torch.bfloat16, B + K + V, "cuda")
@@ -233,7 +240,7 @@ def test_empty_batch_is_a_noop(asd):
     assert out["accepted_len"].numel() == 0
 
 
-def test_one_workspace_serves_many_shapes(asd):
+def test_one_workspace_serves_many_shapes(asd, kernel):
     """The workspace resets itself: one buffer reused across shapes and entry points."""
     ws = asd.Workspace(64, 31, 1, asd.F32)
     rng = np.random.default_rng(8)
@@ -250,6 +257,7 @@ def test_one_workspace_serves_many_shapes(asd):
         o = oracle.verify(b.logits.cpu(), b.draft.cpu().numpy(), np.array([[3.0, 0.0]] * B, np.float32), 1.0, 2,
                           strict=(i % 3 == 0))
         assert_parity(g, o, f"call {i}", ledger=bool(i % 3))
+    assert ws.error() == 0
 
 
 def test_full_size_graph_launch_matches_oracle(asd):
