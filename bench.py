@@ -287,7 +287,7 @@ def run_gpu(args) -> None:
             "hbm_gbs": achieved_gbs, "pct_of_8tbs": achieved_gbs / NOMINAL_HBM_GBS,
             "roofline": {"bound": "hbm", "achieved": achieved_gbs, "peak": pk["hbm_gbs"], "unit": "GB/s",
                          "frac": achieved_gbs / pk["hbm_gbs"], "traffic": recorded_traffic(),
-                         "peak_source": pk["source"], "kernel": "verify_kernel<bf16, asd>",
+                         "peak_source": pk["source"], "kernel": "verify_tma_kernel<bf16, asd>",
                          "algorithmic_bytes_per_launch": bytes_per_launch},
             "clocks": clk,
             "e2e": e2e,
