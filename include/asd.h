@@ -60,7 +60,8 @@ enum {
   ASD_ERR_ALIGN = 6,     /* pointer not aligned as documented */
   ASD_ERR_CUDA = 7,      /* a CUDA call failed (launch or device query) */
   ASD_ERR_DEVICE = 8,    /* the current device cannot run the kernel (not sm_103) */
-  ASD_ERR_TIMEOUT = 9    /* reported by asd_workspace_error: a kernel gave up waiting */
+  ASD_ERR_TIMEOUT = 9,   /* reported by asd_workspace_error: a kernel gave up waiting */
+  ASD_ERR_SCRATCH_LIMIT = 10 /* asd_verify_noalloc: the problem needs more than its scratch */
 };
 
 /* Per-request status bits (status[b]). */
@@ -130,6 +131,37 @@ int asd_verify_strict(const void* logits, int dtype, int B, int K, int V, const 
                       int32_t* accepted_len, int32_t* committed, int32_t* recovery,
                       int32_t* row_argmax, float* row_regret, int32_t* status, void* workspace,
                       size_t workspace_bytes, asd_stream_t stream);
+
+/* Bytes of the fixed device scratch that asd_verify_noalloc uses. */
+#define ASD_NOALLOC_SCRATCH_BYTES (1u << 20)
+
+/*
+ * asd_verify without a caller workspace and without allocating anything: for
+ * callers that may not allocate device memory when they verify (a serving loop
+ * with a fixed device-memory budget, a plug-in whose host framework owns every
+ * device allocation, a latency-bound path where cudaMalloc / cudaFree could
+ * synchronise the device). The paper has no counterpart; it is an interface
+ * convenience around the same computation as asd_verify, with the same
+ * arguments minus the workspace and the same results.
+ *
+ * Scratch: a fixed ASD_NOALLOC_SCRATCH_BYTES array of device memory inside the
+ * library, held by every GPU that loads it until the process exits. A call
+ * whose asd_workspace_size(B, K, V, dtype) exceeds it returns
+ * ASD_ERR_SCRATCH_LIMIT and launches nothing.
+ * Set-up: the first call made with a given device current looks up the
+ * array's device address (cudaGetSymbolAddress); make that first call outside
+ * any stream capture.
+ * Each call clears the part of the array it uses (cudaMemsetAsync on
+ * `stream`) and then launches the verify kernel. Every call on every stream
+ * shares the one array: calls that can overlap on the GPU (different streams,
+ * no ordering between them) race and give wrong results. Order them on one
+ * stream. Allocates nothing: no cudaMalloc, cudaFree or allocating library
+ * call.
+ */
+int asd_verify_noalloc(const void* logits, int dtype, int B, int K, int V, const int32_t* draft,
+                       asd_ledger* ledger, float gate, int cap, int32_t* accepted_len,
+                       int32_t* committed, int32_t* recovery, int32_t* row_argmax,
+                       float* row_regret, int32_t* status, asd_stream_t stream);
 
 /* Human-readable text of a return code. Never NULL. */
 const char* asd_status_string(int code);

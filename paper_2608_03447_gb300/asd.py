@@ -57,6 +57,9 @@ def _declare(lib: ctypes.CDLL) -> ctypes.CDLL:
     lib.asd_verify_strict.restype = i32
     lib.asd_status_string.argtypes = [i32]
     lib.asd_status_string.restype = ctypes.c_char_p
+    if hasattr(lib, "asd_verify_noalloc"):
+        lib.asd_verify_noalloc.argtypes = [vp, i32, i32, i32, i32, vp, vp, f32, i32, vp, vp, vp, vp, vp, vp, vp]
+        lib.asd_verify_noalloc.restype = i32
     if hasattr(lib, "asd_lmhead_workspace_size"):
         lib.asd_lmhead_workspace_size.argtypes = [i32, i32, i32, i32, ctypes.POINTER(sz)]
         lib.asd_lmhead_workspace_size.restype = i32
@@ -184,6 +187,25 @@ def verify(logits: torch.Tensor, draft: torch.Tensor, ledger: torch.Tensor, gate
                            _ptr(o.get("row_argmax")), _ptr(o.get("row_regret")), _ptr(o.get("status")),
                            ws.ptr, ws.nbytes, _stream(stream))
     _check("asd_verify", rc)
+    return o
+
+
+def verify_noalloc(logits: torch.Tensor, draft: torch.Tensor, ledger: torch.Tensor, gate: float, cap: int,
+                   out: dict | None = None, stream=None) -> dict:
+    """asd_verify_noalloc: asd_verify with the library's fixed scratch instead of a workspace.
+
+    For callers that may not allocate device memory while verifying. Calls that
+    may overlap on the GPU share that scratch and must be ordered on one stream.
+    """
+    B, K, V = _shape(logits, draft)
+    if ledger.shape != (B, 2) or ledger.dtype != torch.float32 or not ledger.is_contiguous():
+        raise ValueError("ledger must be a contiguous float32 tensor [B, 2] of (budget, spent)")
+    o = out or alloc_outputs(B, K, logits.device)
+    rc = load().asd_verify_noalloc(_ptr(logits), _dtype_code(logits), B, K, V, _ptr(draft), _ptr(ledger),
+                                   float(gate), int(cap), _ptr(o["accepted_len"]), _ptr(o["committed"]),
+                                   _ptr(o["recovery"]), _ptr(o.get("row_argmax")), _ptr(o.get("row_regret")),
+                                   _ptr(o.get("status")), _stream(stream))
+    _check("asd_verify_noalloc", rc)
     return o
 
 

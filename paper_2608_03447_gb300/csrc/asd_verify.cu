@@ -1246,8 +1246,66 @@ const char* asd_status_string(int code) {
     case ASD_ERR_CUDA: return "CUDA call failed";
     case ASD_ERR_DEVICE: return "the current device cannot run this kernel";
     case ASD_ERR_TIMEOUT: return "a kernel gave up waiting on its own pipeline (outputs incomplete)";
+    case ASD_ERR_SCRATCH_LIMIT:
+      return "problem too large for the built-in scratch of asd_verify_noalloc (use asd_verify)";
     default: return "unknown status code";
   }
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------- allocation-free entry point
+//
+// asd_verify_noalloc: asd_verify for callers that may not allocate device
+// memory at call time (a serving loop with a fixed device-memory budget, a
+// plug-in whose host framework owns every device allocation, a latency-bound
+// path where cudaMalloc/cudaFree could synchronise the device). Its workspace
+// is this file's fixed device array instead of caller memory.
+
+namespace {
+
+// The scratch: every GPU that loads the library holds these bytes until exit.
+static __device__ __align__(256) unsigned char g_noalloc_scratch[ASD_NOALLOC_SCRATCH_BYTES];
+
+// Device address of g_noalloc_scratch on each device, looked up on the first
+// call made with that device current. In host code the symbol itself is only a
+// host-side stand-in: a kernel must be given the looked-up device address.
+int noalloc_scratch(void** out) {
+  constexpr int kMaxDevices = 64;
+  static void* addr[kMaxDevices] = {nullptr};
+  static std::mutex mu;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return ASD_ERR_CUDA;
+  if (dev < 0 || dev >= kMaxDevices) return ASD_ERR_DEVICE;
+  std::lock_guard<std::mutex> g(mu);
+  if (!addr[dev]) {
+    void* ptr = nullptr;
+    if (cudaGetSymbolAddress(&ptr, g_noalloc_scratch) != cudaSuccess || !ptr) return ASD_ERR_CUDA;
+    addr[dev] = ptr;
+  }
+  *out = addr[dev];
+  return ASD_OK;
+}
+
+}  // namespace
+
+extern "C" int asd_verify_noalloc(const void* logits, int dtype, int B, int K, int V,
+                                  const int32_t* draft, asd_ledger* ledger, float gate, int cap,
+                                  int32_t* accepted_len, int32_t* committed, int32_t* recovery,
+                                  int32_t* row_argmax, float* row_regret, int32_t* status,
+                                  asd_stream_t stream) {
+  int rc = check_shape(B, K, V, dtype);
+  if (rc != ASD_OK) return rc;
+  const size_t need = layout_for(B, K).total;
+  if (need > static_cast<size_t>(ASD_NOALLOC_SCRATCH_BYTES)) return ASD_ERR_SCRATCH_LIMIT;
+  if (B == 0) return ASD_OK;
+  void* scratch = nullptr;
+  rc = noalloc_scratch(&scratch);
+  if (rc != ASD_OK) return rc;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  // The array keeps whatever the previous call left; the kernels need the part
+  // they use to start at zero.
+  if (cudaMemsetAsync(scratch, 0, need, s) != cudaSuccess) return ASD_ERR_CUDA;
+  return verify_common(false, logits, dtype, B, K, V, draft, ledger, gate, cap, accepted_len,
+                       committed, recovery, row_argmax, row_regret, status, scratch, need, s);
+}
