@@ -132,6 +132,41 @@ int asd_verify_strict(const void* logits, int dtype, int B, int K, int V, const 
                       int32_t* row_argmax, float* row_regret, int32_t* status, void* workspace,
                       size_t workspace_bytes, asd_stream_t stream);
 
+/*
+ * Fused LM-head + verify (Sec. 3.1 Eq. 1 with Sec. 3.3's remark that the
+ * verifier needs only the top token, the top logit and the draft token's logit,
+ * so no [T, V] logit buffer is needed). The logits z = h W^T are computed on
+ * the tensor cores (bf16 inputs, fp32 accumulation) and reduced on chip; they
+ * are never written to memory. The selection is then the one of asd_verify.
+ *
+ * hidden        [B*(K+1), H] bf16 (as uint16 bits or __nv_bfloat16): the
+ *               target's final hidden state of every row of every block,
+ *               16-byte aligned
+ * weight        [V, H] bf16 LM-head weight, 16-byte aligned
+ * H             hidden size, a multiple of 8 (rows must be 16-byte pitched)
+ * row_top       [B, K+1] the top logit z_j(y*_j) of each row; may be NULL
+ * everything else as in asd_verify; the workspace size comes from
+ * asd_lmhead_workspace_size. Requires a Blackwell (sm_10x) device: other
+ * devices get ASD_ERR_DEVICE.
+ * Precision: the logits are fp32 sums of bf16 products in the tensor core's
+ * order, so ties and near-ties (within about 1e-5 of the row's scale) may
+ * resolve differently from an exact (fp64) evaluation.
+ */
+int asd_lmhead_workspace_size(int B, int K, int V, int H, size_t* bytes);
+int asd_lmhead_verify(const void* hidden, const void* weight, int H, int B, int K, int V,
+                      const int32_t* draft, asd_ledger* ledger, float gate, int cap,
+                      int32_t* accepted_len, int32_t* committed, int32_t* recovery,
+                      int32_t* row_argmax, float* row_regret, float* row_top, int32_t* status,
+                      void* workspace, size_t workspace_bytes, asd_stream_t stream);
+
+/*
+ * The same tensor-core LM-head GEMM writing its fp32 logits [T, V] (row-major,
+ * device memory) instead of reducing them: for callers that need the logits
+ * themselves, and to check the GEMM against an exact evaluation. No workspace.
+ */
+int asd_lmhead_logits(const void* hidden, const void* weight, int H, int T, int V, float* logits,
+                      asd_stream_t stream);
+
 /* Bytes of the fixed device scratch that asd_verify_noalloc uses. */
 #define ASD_NOALLOC_SCRATCH_BYTES (1u << 20)
 

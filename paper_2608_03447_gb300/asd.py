@@ -60,12 +60,13 @@ def _declare(lib: ctypes.CDLL) -> ctypes.CDLL:
     if hasattr(lib, "asd_verify_noalloc"):
         lib.asd_verify_noalloc.argtypes = [vp, i32, i32, i32, i32, vp, vp, f32, i32, vp, vp, vp, vp, vp, vp, vp]
         lib.asd_verify_noalloc.restype = i32
-    if hasattr(lib, "asd_lmhead_workspace_size"):
-        lib.asd_lmhead_workspace_size.argtypes = [i32, i32, i32, i32, ctypes.POINTER(sz)]
-        lib.asd_lmhead_workspace_size.restype = i32
-        lib.asd_lmhead_verify.argtypes = [vp, vp, i32, i32, i32, i32, vp, vp, f32, i32,
-                                          vp, vp, vp, vp, vp, vp, vp, sz, vp]
-        lib.asd_lmhead_verify.restype = i32
+    lib.asd_lmhead_workspace_size.argtypes = [i32, i32, i32, i32, ctypes.POINTER(sz)]
+    lib.asd_lmhead_workspace_size.restype = i32
+    lib.asd_lmhead_verify.argtypes = [vp, vp, i32, i32, i32, i32, vp, vp, f32, i32,
+                                      vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
+    lib.asd_lmhead_verify.restype = i32
+    lib.asd_lmhead_logits.argtypes = [vp, vp, i32, i32, i32, vp, vp]
+    lib.asd_lmhead_logits.restype = i32
     return lib
 
 
@@ -238,3 +239,52 @@ def verify_from_host(logits_host: torch.Tensor, draft_host: torch.Tensor, ledger
     for k in ("accepted_len", "committed", "recovery"):
         host_out[k].copy_(out[k], non_blocking=True)
     return host_out
+
+
+def lmhead_workspace(B: int, K: int, V: int, H: int, device=None, stream=None) -> Workspace:
+    n = ctypes.c_size_t(0)
+    _check("asd_lmhead_workspace_size", load().asd_lmhead_workspace_size(B, K, V, H, ctypes.byref(n)))
+    ws = Workspace.__new__(Workspace)
+    ws.nbytes = n.value
+    ws.buffer = torch.empty(ws.nbytes, dtype=torch.uint8, device=device or "cuda")
+    _check("asd_workspace_init", load().asd_workspace_init(ws.buffer.data_ptr(), ws.nbytes, _stream(stream)))
+    return ws
+
+
+def _lm_shapes(hidden: torch.Tensor, weight: torch.Tensor):
+    for name, t in (("hidden", hidden), ("weight", weight)):
+        if t.dtype != torch.bfloat16 or t.dim() != 2 or not t.is_cuda or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous 2-D bf16 CUDA tensor")
+    if hidden.shape[1] != weight.shape[1]:
+        raise ValueError("hidden and weight must share the hidden size H")
+    return hidden.shape[0], weight.shape[0], hidden.shape[1]
+
+
+def lmhead_verify(hidden: torch.Tensor, weight: torch.Tensor, draft: torch.Tensor, ledger: torch.Tensor,
+                  gate: float, cap: int, workspace: Workspace | None = None, out: dict | None = None,
+                  stream=None) -> dict:
+    """asd_lmhead_verify: logits = hidden @ weight.T on the tensor cores, reduced on chip, then Alg. 1."""
+    T, V, H = _lm_shapes(hidden, weight)
+    B, K = draft.shape
+    if T != B * (K + 1):
+        raise ValueError("hidden must hold B*(K+1) rows")
+    ws = workspace or lmhead_workspace(B, K, V, H, hidden.device, stream)
+    o = out or alloc_outputs(B, K, hidden.device)
+    if "row_top" not in o:
+        o["row_top"] = torch.empty(B, K + 1, dtype=torch.float32, device=hidden.device)
+    rc = load().asd_lmhead_verify(_ptr(hidden), _ptr(weight), H, B, K, V, _ptr(draft), _ptr(ledger), float(gate),
+                                  int(cap), _ptr(o["accepted_len"]), _ptr(o["committed"]), _ptr(o["recovery"]),
+                                  _ptr(o.get("row_argmax")), _ptr(o.get("row_regret")), _ptr(o.get("row_top")),
+                                  _ptr(o.get("status")), ws.ptr, ws.nbytes, _stream(stream))
+    _check("asd_lmhead_verify", rc)
+    return o
+
+
+def lmhead_logits(hidden: torch.Tensor, weight: torch.Tensor, out: torch.Tensor | None = None,
+                  stream=None) -> torch.Tensor:
+    """asd_lmhead_logits: the same tensor-core GEMM, writing the fp32 logits [T, V]."""
+    T, V, H = _lm_shapes(hidden, weight)
+    o = out if out is not None else torch.empty(T, V, dtype=torch.float32, device=hidden.device)
+    _check("asd_lmhead_logits", load().asd_lmhead_logits(_ptr(hidden), _ptr(weight), H, T, V, _ptr(o),
+                                                         _stream(stream)))
+    return o

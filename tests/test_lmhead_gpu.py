@@ -1,0 +1,159 @@
+"""Fused LM-head + verify (asd_lmhead_verify, asd_lmhead_logits) against the fp64 oracle.
+
+The tensor cores accumulate bf16 products in fp32, so the comparison follows
+the stated tolerance: logits within 2e-2 (absolute) of the fp64 oracle, and
+decisions (argmax, accepted length, committed and recovery tokens) bit-exact
+wherever they are decided by a margin larger than the arithmetic can move:
+a row's argmax where its top-2 gap exceeds 5e-2; a request's selection where
+every row has such a gap, every mismatch has |r/q - g| > 5e-2 and every
+budget test has |fl(s + C) - B| > 4e-2 per accumulated mismatch.
+"""
+import concurrent.futures as cf
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import oracle
+from paper_2608_03447_gb300 import inputs
+
+pytestmark = pytest.mark.gpu
+LOGIT_TOL = 2e-2
+MARGIN = 5e-2
+
+
+def oracle_logits(hidden, weight, tokens, threads=16):
+    """fp64 oracle logits of the given token rows (one thread per token; ctypes releases the GIL)."""
+    h = hidden.cpu()
+    w = weight.cpu()
+    tokens = list(tokens)
+    with cf.ThreadPoolExecutor(max_workers=threads) as pool:
+        parts = list(pool.map(lambda t: oracle.lmhead_logits(h, w, np.array([t], np.int32)), tokens))
+    z64 = np.concatenate([p[0] for p in parts])
+    z32 = np.concatenate([p[1] for p in parts])
+    return z64, z32
+
+
+def top2_gap(z64):
+    part = np.partition(z64, -2, axis=1)
+    return part[:, -1] - part[:, -2]
+
+
+def eligible(o, z64_req, K, gate, cap, budget, spent):
+    """Is this request's selection decided by margins larger than the tolerance?"""
+    if np.any(top2_gap(z64_req) <= MARGIN):
+        return False
+    y = o["row_argmax"]
+    r = o["row_regret"]
+    x_match = o["committed"]  # unused; decisions come from y and r
+    C, N = np.float32(0.0), 0
+    for j in range(K):
+        if o["draft"][j] == y[j]:
+            continue
+        if abs(float(r[j]) / (K - j) - gate) <= MARGIN:
+            return False
+        C = np.float32(C + r[j])
+        N += 1
+        if abs(float(np.float32(spent + C)) - budget) <= 4e-2 * N:
+            return False
+        if not (np.float32(r[j]) / np.float32(K - j) <= gate and np.float32(spent + C) <= budget and N <= cap):
+            break
+    return True
+
+
+def compare(out, z64, z32, draft, tokens, B, K, gate, cap, budget):
+    """Check the GPU outputs of the requests whose rows are `tokens` (whole requests) against the oracle."""
+    K1 = K + 1
+    reqs = sorted(set(t // K1 for t in tokens))
+    g_top = out["row_top"].cpu().numpy().reshape(-1)
+    g_arg = out["row_argmax"].cpu().numpy().reshape(-1)
+    g_reg = out["row_regret"].cpu().numpy().reshape(B, K)
+    g_acc = out["accepted_len"].cpu().numpy()
+    g_com = out["committed"].cpu().numpy()
+    g_rec = out["recovery"].cpu().numpy()
+    x = draft.cpu().numpy()
+    pos = {t: i for i, t in enumerate(tokens)}
+    n_eligible = 0
+    for b in reqs:
+        rows = [pos[b * K1 + j] for j in range(K1)]
+        zr32 = z32[rows][None]
+        o = oracle.verify(zr32, x[b:b + 1], np.array([[budget, 0.0]], np.float32), gate, cap)
+        o1 = {k: v[0] for k, v in o.items()}
+        o1["draft"] = x[b]
+        zmax = z64[rows].max(axis=1)
+        assert np.all(np.abs(g_top[b * K1:(b + 1) * K1] - zmax) <= LOGIT_TOL), f"request {b}: top logit"
+        gaps = top2_gap(z64[rows])
+        decided = gaps > MARGIN
+        assert np.array_equal(g_arg[b * K1:(b + 1) * K1][decided], o1["row_argmax"][decided]), f"request {b}: argmax"
+        for j in range(K):
+            if 0 <= x[b, j]:
+                zx = z64[rows[j], x[b, j]]
+                assert abs(g_reg[b, j] - (zmax[j] - zx)) <= 2 * LOGIT_TOL, f"request {b} row {j}: regret"
+        if eligible(o1, z64[rows], K, gate, cap, budget, 0.0):
+            n_eligible += 1
+            assert g_acc[b] == o1["accepted_len"], f"request {b}: accepted length"
+            assert np.array_equal(g_com[b], o1["committed"]), f"request {b}: committed"
+            assert g_rec[b] == o1["recovery"], f"request {b}: recovery"
+    return n_eligible, len(reqs)
+
+
+@pytest.mark.parametrize("T,H,V", [(36, 512, 1000), (300, 136, 777), (130, 64, 256), (129, 5120, 2100)])
+def test_lmhead_logits_match_fp64(asd, T, H, V):
+    g = torch.Generator(device="cuda").manual_seed(T * 7 + H + V)
+    h = torch.randn(T, H, generator=g, device="cuda").to(torch.bfloat16)
+    w = (0.02 * torch.randn(V, H, generator=g, device="cuda")).to(torch.bfloat16)
+    z = asd.lmhead_logits(h, w)
+    torch.cuda.synchronize()
+    z64, _ = oracle_logits(h, w, range(T))
+    err = np.abs(z.cpu().numpy().astype(np.float64) - z64)
+    assert err.max() <= LOGIT_TOL, f"max |logit - fp64| = {err.max()}"
+    assert err.max() <= 1e-3, f"fp32 accumulation should be far inside the tolerance: {err.max()}"
+
+
+@pytest.mark.parametrize("B,K,H,V", [(4, 8, 512, 4096), (16, 7, 1024, 3000), (3, 0, 256, 999)])
+def test_lmhead_verify_small(asd, B, K, H, V):
+    inp = inputs.gen_lmhead(B, K, H, V, 4000 + B + K + H, "cuda")
+    led = asd.make_ledger(B, 8.0)
+    out = asd.lmhead_verify(inp.hidden, inp.weight, inp.draft, led, 1.0, 2)
+    torch.cuda.synchronize()
+    T = B * (K + 1)
+    z64, z32 = oracle_logits(inp.hidden, inp.weight, range(T))
+    n_ok, n = compare(out, z64, z32, inp.draft, list(range(T)), B, K, 1.0, 2, 8.0)
+    assert n_ok >= n // 2, f"too few requests decided by margin ({n_ok}/{n}); the workload is too tie-heavy"
+
+
+def test_lmhead_strict_budget_zero_matches_argmax(asd):
+    """Budget 0: the fused verify is exact greedy verification on its own argmaxes."""
+    B, K, H, V = 8, 8, 512, 2048
+    inp = inputs.gen_lmhead(B, K, H, V, 77, "cuda")
+    led = asd.make_ledger(B, 0.0)
+    out = asd.lmhead_verify(inp.hidden, inp.weight, inp.draft, led, 1.0, 2)
+    torch.cuda.synchronize()
+    y = out["row_argmax"].cpu().numpy()
+    x = inp.draft.cpu().numpy()
+    for b in range(B):
+        a = next((j for j in range(K) if x[b, j] != y[b, j]), K)
+        assert out["accepted_len"][b].item() == a
+        assert out["recovery"][b].item() == y[b, a]
+    assert torch.equal(led.cpu(), torch.zeros(B, 2))
+
+
+def test_lmhead_full_size_sampled(asd):
+    """B=64, K=8, H=5120, V=151936 (Qwen3-14B LM head shape); the fp64 oracle checks 3 whole requests."""
+    cfg = inputs.CONFIGS[4]
+    B, K, H, V = cfg["B"], cfg["K"], cfg["H"], cfg["V"]
+    inp = inputs.gen_lmhead(B, K, H, V, inputs.seed_for(4), "cuda")
+    led = asd.make_ledger(B, cfg["budget"])
+    ws = asd.lmhead_workspace(B, K, V, H)
+    for _ in range(2):  # the second call reuses the workspace and carries the ledger
+        led.copy_(asd.make_ledger(B, cfg["budget"]))
+        out = asd.lmhead_verify(inp.hidden, inp.weight, inp.draft, led, cfg["gate"], cfg["cap"], workspace=ws)
+    torch.cuda.synchronize()
+    assert ws.error() == 0
+    K1 = K + 1
+    reqs = [0, 31, 63]
+    tokens = [b * K1 + j for b in reqs for j in range(K1)]
+    z64, z32 = oracle_logits(inp.hidden, inp.weight, tokens)
+    n_ok, n = compare(out, z64, z32, inp.draft, tokens, B, K, cfg["gate"], cfg["cap"], cfg["budget"])
+    assert n_ok >= 1
