@@ -185,6 +185,25 @@ def dist_env():
     return rank, world, local
 
 
+def rank_config(rank: int) -> int:
+    """Seed family of a rank's own batch: ranks verify disjoint requests (weak scaling)."""
+    return 1 + 100 * rank
+
+
+def max_over_ranks(value: float, device, world: int) -> float:
+    """The job's time is its slowest rank's (all_reduce MAX over the process group)."""
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    if world > 1:
+        import torch.distributed as dist
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rows_per_s(world: int, rows_per_step: int, steps: int, seconds: float) -> float:
+    """Whole-job throughput: the rows every rank verified over the slowest rank's time."""
+    return world * rows_per_step * steps / seconds
+
+
 def run_reference(args) -> None:
     """The CPU oracle as it stands, on the host cores: one full block of the workload per step."""
     import concurrent.futures as cf
@@ -275,7 +294,7 @@ def run_gpu(args) -> None:
         dist.init_process_group("nccl", device_id=dev)
     asd.load()
 
-    wl = VerifyWorkload(B, K, V, torch.bfloat16, GATE, CAP, BUDGET, config=1 + 100 * rank, device=dev)
+    wl = VerifyWorkload(B, K, V, torch.bfloat16, GATE, CAP, BUDGET, config=rank_config(rank), device=dev)
     steps, warmup = args.steps, args.warmup
     G = min(steps, 512)
     graph_full = wl.capture(G, first=0)
@@ -311,14 +330,10 @@ def run_gpu(args) -> None:
     barrier()
     clocks.mark_end()
     clk = clocks.stop()
-    ms = start.elapsed_time(end)
-    t = torch.tensor([ms], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    ms_max = float(t.item())
+    ms_max = max_over_ranks(start.elapsed_time(end), dev, world)
     sec_per_step = ms_max / 1e3 / steps
     rows_per_step = B * (K + 1)
-    value = world * rows_per_step / sec_per_step
+    value = job_rows_per_s(world, rows_per_step, steps, ms_max / 1e3)
     bytes_per_launch = wl.bytes_per_step
     achieved_gbs = bytes_per_launch / sec_per_step / 1e9
 
@@ -378,14 +393,10 @@ def run_e2e(wl, dev, steps: int, world: int) -> dict:
                              wl.workspace, wl.out, host_out)
     end.record(stream)
     end.synchronize()
-    ms = start.elapsed_time(end)
-    t = torch.tensor([ms], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    sec = float(t.item()) / 1e3
+    sec = max_over_ranks(start.elapsed_time(end), dev, world) / 1e3
     h2d = host_logits[0].numel() * host_logits[0].element_size() + host_draft[0].numel() * 4
     d2h = sum(v.numel() * v.element_size() for v in host_out.values())
-    return {"value": world * steps * B * (K + 1) / sec, "unit": "rows/s", "h2d_bytes_per_step": h2d,
+    return {"value": job_rows_per_s(world, B * (K + 1), steps, sec), "unit": "rows/s", "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "steps": steps}
 
 
