@@ -198,6 +198,26 @@ int asd_verify_noalloc(const void* logits, int dtype, int B, int K, int V, const
                        int32_t* committed, int32_t* recovery, int32_t* row_argmax,
                        float* row_regret, int32_t* status, asd_stream_t stream);
 
+/*
+ * Several sequential draft blocks of the same B requests in one call: block i
+ * of request b is verified with the ledger left by block i-1 (Sec. 3.2: the
+ * ledger (B, s) persists across decoding rounds). The result is bit for bit
+ * that of nblk asd_verify calls made in order, block 0 first.
+ *
+ * logits        [nblk, B, K+1, V]; draft [nblk, B, K]; ledger [B] in/out
+ * accepted_len, recovery, status  [nblk, B]; committed, row_argmax [nblk, B, K+1];
+ * row_regret    [nblk, B, K]
+ * workspace     asd_blocks_workspace_size(nblk, B, K, V, dtype) bytes
+ * The logits of all blocks stream in one pass; only each request's selection
+ * runs block after block, with the ledger in registers.
+ */
+int asd_blocks_workspace_size(int nblk, int B, int K, int V, int dtype, size_t* bytes);
+int asd_verify_blocks(const void* logits, int dtype, int nblk, int B, int K, int V,
+                      const int32_t* draft, asd_ledger* ledger, float gate, int cap,
+                      int32_t* accepted_len, int32_t* committed, int32_t* recovery,
+                      int32_t* row_argmax, float* row_regret, int32_t* status, void* workspace,
+                      size_t workspace_bytes, asd_stream_t stream);
+
 /* Human-readable text of a return code. Never NULL. */
 const char* asd_status_string(int code);
 

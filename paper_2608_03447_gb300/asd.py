@@ -57,6 +57,11 @@ def _declare(lib: ctypes.CDLL) -> ctypes.CDLL:
     lib.asd_verify_strict.restype = i32
     lib.asd_status_string.argtypes = [i32]
     lib.asd_status_string.restype = ctypes.c_char_p
+    lib.asd_blocks_workspace_size.argtypes = [i32, i32, i32, i32, i32, ctypes.POINTER(sz)]
+    lib.asd_blocks_workspace_size.restype = i32
+    lib.asd_verify_blocks.argtypes = [vp, i32, i32, i32, i32, i32, vp, vp, f32, i32, vp, vp, vp, vp, vp, vp, vp, sz,
+                                      vp]
+    lib.asd_verify_blocks.restype = i32
     if hasattr(lib, "asd_verify_noalloc"):
         lib.asd_verify_noalloc.argtypes = [vp, i32, i32, i32, i32, vp, vp, f32, i32, vp, vp, vp, vp, vp, vp, vp]
         lib.asd_verify_noalloc.restype = i32
@@ -288,3 +293,41 @@ def lmhead_logits(hidden: torch.Tensor, weight: torch.Tensor, out: torch.Tensor 
     _check("asd_lmhead_logits", load().asd_lmhead_logits(_ptr(hidden), _ptr(weight), H, T, V, _ptr(o),
                                                          _stream(stream)))
     return o
+
+
+def blocks_workspace(nblk: int, B: int, K: int, V: int, dtype: int, device=None, stream=None) -> Workspace:
+    n = ctypes.c_size_t(0)
+    _check("asd_blocks_workspace_size", load().asd_blocks_workspace_size(nblk, B, K, V, dtype, ctypes.byref(n)))
+    ws = Workspace.__new__(Workspace)
+    ws.nbytes = n.value
+    ws.buffer = torch.empty(max(ws.nbytes, 1), dtype=torch.uint8, device=device or "cuda")
+    _check("asd_workspace_init", load().asd_workspace_init(ws.buffer.data_ptr(), ws.nbytes, _stream(stream)))
+    return ws
+
+
+def verify_blocks(logits: torch.Tensor, draft: torch.Tensor, ledger: torch.Tensor, gate: float, cap: int,
+                  workspace: Workspace | None = None, out: dict | None = None, stream=None) -> dict:
+    """asd_verify_blocks: nblk sequential blocks of the same requests in one call.
+
+    logits [nblk, B, K+1, V], draft [nblk, B, K], ledger [B, 2]; outputs carry a
+    leading nblk dimension.
+    """
+    if logits.dim() != 4 or not logits.is_cuda or not logits.is_contiguous():
+        raise ValueError("logits must be a contiguous CUDA tensor [nblk, B, K+1, V]")
+    nblk, B, K1, V = logits.shape
+    K = K1 - 1
+    if draft.shape != (nblk, B, K) or draft.dtype != torch.int32 or not draft.is_contiguous():
+        raise ValueError("draft must be a contiguous int32 tensor [nblk, B, K]")
+    if ledger.shape != (B, 2) or ledger.dtype != torch.float32 or not ledger.is_contiguous():
+        raise ValueError("ledger must be a contiguous float32 tensor [B, 2] of (budget, spent)")
+    code = _dtype_code(logits)
+    ws = workspace or blocks_workspace(nblk, B, K, V, code, logits.device, stream)
+    if out is None:
+        flat = alloc_outputs(nblk * B, K, logits.device)
+        out = {k: v.view(nblk, B, *v.shape[1:]) for k, v in flat.items()}
+    rc = load().asd_verify_blocks(_ptr(logits), code, nblk, B, K, V, _ptr(draft), _ptr(ledger), float(gate),
+                                  int(cap), _ptr(out["accepted_len"]), _ptr(out["committed"]), _ptr(out["recovery"]),
+                                  _ptr(out.get("row_argmax")), _ptr(out.get("row_regret")), _ptr(out.get("status")),
+                                  ws.ptr, ws.nbytes, _stream(stream))
+    _check("asd_verify_blocks", rc)
+    return out

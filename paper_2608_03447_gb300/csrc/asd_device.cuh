@@ -33,9 +33,10 @@ struct VerifyParams {
   unsigned long long* row_key;  // [B*(K+1)] running (value, index) key, zero between calls
   float* draft_logit;           // [B*(K+1)] z_j(x_j), written by the segment holding x_j
   unsigned long long* done;     // [B] elements finished, zero between calls
-  unsigned int* flags;          // [B] ASD_STATUS_NAN_LOGIT bits, zero between calls
+  unsigned int* flags;          // [nblk*B] ASD_STATUS_NAN_LOGIT bits, zero between calls
   unsigned int* error;          // sticky: ASD_ERR_TIMEOUT when a pipeline wait gave up
   float* row_top;               // [B*(K+1)] z_j(y*_j), or NULL (written by the fused LM-head path)
+  int nblk;                     // sequential blocks of the same B requests (block i = requests i*B ..)
 };
 
 // ---------------------------------------------------------------- element access
@@ -103,47 +104,66 @@ __device__ __forceinline__ bool ledger_invalid(float budget, float spent) {
   return budget != budget || spent != spent || budget < 0.0f || spent < 0.0f || spent > budget;
 }
 
-template <typename T, bool kStrict>
-__device__ void select_request(const VerifyParams& p, int b, int lane) {
+// What one block's selection reads from the workspace for one request
+// (lane j: target row j); loaded ahead of use.
+struct BlockInputs {
+  unsigned long long key;  // row j's (value, index) key
+  int x;                   // draft token j (lanes < K)
+  float zx;                // z_j(x_j) (lanes < K)
+  unsigned flags;          // the block's status bits (every lane)
+};
+
+__device__ __forceinline__ BlockInputs load_block(const VerifyParams& p, long long vb, int lane) {
   const int K = p.K, K1 = p.K + 1;
-  const long long row = static_cast<long long>(b) * K1 + lane;
-  const T* z = static_cast<const T*>(p.logits);
-
-  unsigned long long key = 0;
-  int x = -1;
-  float zx = 0.0f;
-  if (lane < K1) key = atomicExch(&p.row_key[row], 0ull);
+  const long long row = vb * K1 + lane;
+  BlockInputs in;
+  in.key = 0;
+  in.x = -1;
+  in.zx = 0.0f;
+  in.flags = 0;
+  if (lane < K1) {
+    in.key = __ldcg(&p.row_key[row]);
+    p.row_key[row] = 0ull;  // the whole workspace is zero again after every call
+  }
   if (lane < K) {
-    x = p.draft[static_cast<long long>(b) * K + lane];
-    zx = __ldcg(&p.draft_logit[row]);
-    p.draft_logit[row] = 0.0f;  // the whole workspace is zero again after every call
+    in.x = p.draft[vb * K + lane];
+    in.zx = __ldcg(&p.draft_logit[row]);
+    p.draft_logit[row] = 0.0f;
   }
-  unsigned flags = 0;
-  float budget = 0.0f, spent = 0.0f;
   if (lane == 0) {
-    flags = atomicExch(&p.flags[b], 0u);
-    if (!kStrict) {
-      budget = p.ledger[b].budget;
-      spent = p.ledger[b].spent;
-    }
+    in.flags = __ldcg(&p.flags[vb]);
+    p.flags[vb] = 0u;
   }
-  flags = __shfl_sync(kFull, flags, 0);
-  budget = __shfl_sync(kFull, budget, 0);
-  spent = __shfl_sync(kFull, spent, 0);
+  in.flags = __shfl_sync(kFull, in.flags, 0);
+  return in;
+}
 
-  const int y = key == 0 ? 0 : static_cast<int>(0xffffffffu - static_cast<uint32_t>(key));
+// Alg. 1 for block vb of one request, given the request's ledger (budget,
+// spent): writes the block's outputs and advances `spent` (Eq. 13) unless the
+// block is strict, zero-budget or flagged.
+template <typename T, bool kStrict>
+__device__ __forceinline__ void select_block(const VerifyParams& p, long long vb, const BlockInputs& in,
+                                             float budget, float& spent, bool& wrote, int lane) {
+  const int K = p.K, K1 = p.K + 1;
+  const long long row = vb * K1 + lane;
+  const T* z = static_cast<const T*>(p.logits);
+  unsigned flags = in.flags;
+  const int x = in.x;
+
+  const int y = in.key == 0 ? 0 : static_cast<int>(0xffffffffu - static_cast<uint32_t>(in.key));
   const bool valid_x = lane < K && x >= 0 && x < p.V;
   if (__any_sync(kFull, lane < K && !valid_x)) flags |= ASD_STATUS_DRAFT_RANGE;
 
   // Eq. 3: r_j = z_j(y*_j) - z_j(x_j). The key holds the maximum exactly, except
   // that it folds -0 onto +0; a zero maximum is re-read to keep its sign (when
   // the logits are in memory: the fused LM-head path passes none).
+  const float top = ordered_value(static_cast<uint32_t>(in.key >> 32));
   float r = 0.0f;
   if (lane < K) {
     if (valid_x) {
-      float top = ordered_value(static_cast<uint32_t>(key >> 32));
-      if (top == 0.0f && z) top = Elem<T>::load(z, row * p.V + y);
-      r = __fsub_rn(top, zx);
+      float t = top;
+      if (t == 0.0f && z) t = Elem<T>::load(z, row * p.V + y);
+      r = __fsub_rn(t, in.zx);
     } else {
       r = __int_as_float(0x7fc00000);
     }
@@ -153,8 +173,6 @@ __device__ void select_request(const VerifyParams& p, int b, int lane) {
   if (!kStrict && ledger_invalid(budget, spent)) flags |= ASD_STATUS_BAD_LEDGER;
 
   int a;
-  bool write_ledger = false;
-  float new_spent = spent;
   if (flags) {
     a = 0;
   } else if (kStrict || budget == 0.0f) {
@@ -180,22 +198,47 @@ __device__ void select_request(const VerifyParams& p, int b, int lane) {
       C = C_next;
       N = N_next;
     }
-    new_spent = __fadd_rn(spent, C);  // Eq. 13
-    write_ledger = true;
+    spent = __fadd_rn(spent, C);  // Eq. 13
+    wrote = true;
   }
   const int ya = __shfl_sync(kFull, y, a);
 
   if (lane < K1) {
     if (p.row_argmax) p.row_argmax[row] = y;
     p.committed[row] = lane < a ? x : (lane == a ? ya : -1);
+    if (p.row_top) p.row_top[row] = top;
   }
-  if (lane < K && p.row_regret) p.row_regret[static_cast<long long>(b) * K + lane] = r;
-  if (lane < K1 && p.row_top) p.row_top[row] = ordered_value(static_cast<uint32_t>(key >> 32));
+  if (lane < K && p.row_regret) p.row_regret[vb * K + lane] = r;
   if (lane == 0) {
-    p.accepted_len[b] = a;
-    p.recovery[b] = ya;
-    if (p.status) p.status[b] = static_cast<int32_t>(flags);
-    if (write_ledger) p.ledger[b].spent = new_spent;
+    p.accepted_len[vb] = a;
+    p.recovery[vb] = ya;
+    if (p.status) p.status[vb] = static_cast<int32_t>(flags);
+  }
+}
+
+// The selection of request b over its p.nblk blocks in order (block i is the
+// virtual request i * B + b): the ledger is read once, carried in registers
+// from block to block, and written once. Runs in one warp.
+template <typename T, bool kStrict>
+__device__ void select_request(const VerifyParams& p, int b, int lane) {
+  float budget = 0.0f, spent = 0.0f;
+  if (!kStrict && lane == 0) {
+    budget = p.ledger[b].budget;
+    spent = p.ledger[b].spent;
+  }
+  budget = __shfl_sync(kFull, budget, 0);
+  spent = __shfl_sync(kFull, spent, 0);
+  bool wrote = false;
+  BlockInputs cur = load_block(p, b, lane);
+  for (int i = 0; i < p.nblk; ++i) {
+    const long long vb = static_cast<long long>(i) * p.B + b;
+    BlockInputs next = cur;
+    if (i + 1 < p.nblk) next = load_block(p, vb + p.B, lane);  // in flight while this block is selected
+    select_block<T, kStrict>(p, vb, cur, budget, spent, wrote, lane);
+    cur = next;
+  }
+  if (lane == 0) {
+    if (wrote) p.ledger[b].spent = spent;
     p.done[b] = 0ull;
   }
 }

@@ -493,6 +493,7 @@ int asd_lmhead_verify(const void* hidden, const void* weight, int H, int B, int 
   p.flags = reinterpret_cast<unsigned int*>(ws + l.flags);
   p.error = reinterpret_cast<unsigned int*>(ws + l.error);
   p.row_top = row_top;
+  p.nblk = 1;
   return launch_lmhead<false, false>(hidden, weight, H, B * (K + 1), p, nullptr,
                                      reinterpret_cast<cudaStream_t>(stream));
 }
@@ -507,6 +508,7 @@ int asd_lmhead_logits(const void* hidden, const void* weight, int H, int T, int 
   VerifyParams p = {};
   p.V = V;
   p.K = 0;
+  p.nblk = 1;
   return launch_lmhead<false, true>(hidden, weight, H, T, p, logits, reinterpret_cast<cudaStream_t>(stream));
 }
 

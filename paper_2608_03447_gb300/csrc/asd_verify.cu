@@ -189,7 +189,8 @@ __global__ void ASD_VERIFY_BOUNDS verify_kernel(const VerifyParams p) {
 
   const T* z = static_cast<const T*>(p.logits);
   const int V = p.V, K = p.K, K1 = p.K + 1;
-  const unsigned long long request_elems = static_cast<unsigned long long>(K1) * V;
+  // counters are per request; a request is complete when all p.nblk of its blocks are
+  const unsigned long long request_elems = static_cast<unsigned long long>(K1) * V * p.nblk;
 
   long long row = lo / V;
   int pending_b = static_cast<int>(row / K1);
@@ -203,16 +204,16 @@ __global__ void ASD_VERIFY_BOUNDS verify_kernel(const VerifyParams p) {
     int x = -1;
     if (j < K) x = __ldg(p.draft + static_cast<long long>(b) * K + j);  // issued before the stream
 
-    if (b != pending_b) {  // finished this warp's share of request pending_b
+    if (b != pending_b) {  // finished this warp's share of block-request pending_b
       bool last = false;
       if (lane == 0) {
         __threadfence();
-        const unsigned long long old = atomicAdd(&p.done[pending_b], pending_n);
+        const unsigned long long old = atomicAdd(&p.done[pending_b % p.B], pending_n);
         last = old + pending_n == request_elems;
       }
       if (__shfl_sync(kFull, last, 0)) {
         __threadfence();
-        select_request<T, kStrict>(p, pending_b, lane);
+        select_request<T, kStrict>(p, pending_b % p.B, lane);
       }
       pending_b = b;
       pending_n = 0;
@@ -233,12 +234,12 @@ __global__ void ASD_VERIFY_BOUNDS verify_kernel(const VerifyParams p) {
   bool last = false;
   if (lane == 0) {
     __threadfence();
-    const unsigned long long old = atomicAdd(&p.done[pending_b], pending_n);
+    const unsigned long long old = atomicAdd(&p.done[pending_b % p.B], pending_n);
     last = old + pending_n == request_elems;
   }
   if (__shfl_sync(kFull, last, 0)) {
     __threadfence();
-    select_request<T, kStrict>(p, pending_b, lane);
+    select_request<T, kStrict>(p, pending_b % p.B, lane);
   }
 }
 
@@ -383,7 +384,7 @@ __device__ __forceinline__ int draft_of_row(const VerifyParams& p, long long row
   const int K1 = p.K + 1;
   const long long b = row / K1;
   const int j = static_cast<int>(row - b * K1);
-  if (j >= p.K || b >= p.B) return -1;
+  if (j >= p.K || b >= static_cast<long long>(p.B) * p.nblk) return -1;  // b: block-request
   return __ldg(p.draft + b * p.K + j);
 }
 
@@ -696,8 +697,8 @@ __global__ void __launch_bounds__(kTmaThreads, 1)
     for (long long b = b_first + warp; b <= b_last; b += kTmaConsumers + 1) {
       const long long r0 = b * rv > cta_lo ? b * rv : cta_lo;
       const long long r1 = (b + 1) * rv < cta_hi ? (b + 1) * rv : cta_hi;
-      finish_request<T, kStrict>(p, static_cast<int>(b), static_cast<unsigned long long>(r1 - r0),
-                                 static_cast<unsigned long long>(rv), lane);
+      finish_request<T, kStrict>(p, static_cast<int>(b % p.B), static_cast<unsigned long long>(r1 - r0),
+                                 static_cast<unsigned long long>(rv) * p.nblk, lane);
     }
   }
 }
@@ -851,17 +852,18 @@ int verify_common(bool strict, const void* logits, int dtype, int B, int K, int 
                   const int32_t* draft, asd_ledger* ledger, float gate, int cap,
                   int32_t* accepted_len, int32_t* committed, int32_t* recovery,
                   int32_t* row_argmax, float* row_regret, int32_t* status, void* workspace,
-                  size_t workspace_bytes, cudaStream_t stream) {
+                  size_t workspace_bytes, cudaStream_t stream, int nblk = 1) {
   int rc = check_shape(B, K, V, dtype);
   if (rc != ASD_OK) return rc;
-  if (B == 0) return ASD_OK;
+  if (nblk < 0 || (nblk > 0 && B > INT32_MAX / nblk)) return ASD_ERR_SHAPE;
+  if (B == 0 || nblk == 0) return ASD_OK;
   if (!logits || !accepted_len || !committed || !recovery || !workspace) return ASD_ERR_NULL;
   if (K > 0 && !draft) return ASD_ERR_NULL;
   if (!strict) {
     if (!ledger) return ASD_ERR_NULL;
     if (gate != gate || gate < 0.0f || cap < 0) return ASD_ERR_CONTROL;
   }
-  const WorkspaceLayout l = layout_for(B, K);
+  const WorkspaceLayout l = layout_for(nblk * B, K);
   if (workspace_bytes < l.total) return ASD_ERR_WORKSPACE;
   if (reinterpret_cast<uintptr_t>(workspace) % 16 != 0) return ASD_ERR_ALIGN;
   char* ws = static_cast<char*>(workspace);
@@ -871,7 +873,8 @@ int verify_common(bool strict, const void* logits, int dtype, int B, int K, int 
   p.B = B;
   p.K = K;
   p.V = V;
-  p.total = static_cast<long long>(B) * (K + 1) * V;
+  p.nblk = nblk;
+  p.total = static_cast<long long>(nblk) * B * (K + 1) * V;
   p.head = 0;
   p.per_warp = 0;
   p.draft = draft;
@@ -942,6 +945,24 @@ int asd_verify_strict(const void* logits, int dtype, int B, int K, int V, const 
   return verify_common(true, logits, dtype, B, K, V, draft, nullptr, 0.0f, 0, accepted_len,
                        committed, recovery, row_argmax, row_regret, status, workspace,
                        workspace_bytes, reinterpret_cast<cudaStream_t>(stream));
+}
+
+int asd_blocks_workspace_size(int nblk, int B, int K, int V, int dtype, size_t* bytes) {
+  if (!bytes) return ASD_ERR_NULL;
+  const int rc = check_shape(B, K, V, dtype);
+  if (rc != ASD_OK) return rc;
+  if (nblk < 0 || (nblk > 0 && B > INT32_MAX / nblk)) return ASD_ERR_SHAPE;
+  *bytes = layout_for(nblk * B, K).total;
+  return ASD_OK;
+}
+
+int asd_verify_blocks(const void* logits, int dtype, int nblk, int B, int K, int V, const int32_t* draft,
+                      asd_ledger* ledger, float gate, int cap, int32_t* accepted_len, int32_t* committed,
+                      int32_t* recovery, int32_t* row_argmax, float* row_regret, int32_t* status,
+                      void* workspace, size_t workspace_bytes, asd_stream_t stream) {
+  return verify_common(false, logits, dtype, B, K, V, draft, ledger, gate, cap, accepted_len, committed,
+                       recovery, row_argmax, row_regret, status, workspace, workspace_bytes,
+                       reinterpret_cast<cudaStream_t>(stream), nblk);
 }
 
 const char* asd_status_string(int code) {
