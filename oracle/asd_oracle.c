@@ -256,3 +256,35 @@ void oracle_lmhead_logits(const uint16_t* h, const uint16_t* W, int H, int V,
     }
   }
 }
+
+/*
+ * Eq. 4, the verifier-side opportunity rate, as counts: over every mismatch
+ * position (x, i) of the given blocks (1-based i with x_i != y*_i, i <= K),
+ *   num[t][u] = #{ (x, i) : r_i <= tau[t], i + p[u] <= K, x_l = y*_l for l = i+1 .. i+p[u] }
+ *   *den      = |M|, the number of mismatch positions.
+ * Omega(tau, p) = num / den. Blocks with a non-zero status word (when given)
+ * are skipped. Counts are added to num / den (accumulated over calls).
+ *   row_argmax [n, K+1], draft [n, K], row_regret [n, K], status [n] or NULL
+ */
+void oracle_opportunity(const int32_t* row_argmax, const int32_t* draft, const float* row_regret,
+                        const int32_t* status, int n, int K, const float* tau, int ntau,
+                        const int32_t* p, int np, long long* num, long long* den) {
+  for (int b = 0; b < n; b++) {
+    if (status && status[b] != 0) continue;
+    const int32_t* y = row_argmax + (int64_t)b * (K + 1);
+    const int32_t* x = draft + (int64_t)b * K;
+    const float* r = row_regret + (int64_t)b * K;
+    for (int i = 1; i <= K; i++) {           /* 1-based position, as in Eq. 4 */
+      if (x[i - 1] == y[i - 1]) continue;    /* only mismatches belong to M */
+      *den += 1;
+      for (int u = 0; u < np; u++) {
+        int reusable = i + p[u] <= K;
+        for (int l = i + 1; reusable && l <= i + p[u]; l++)
+          if (x[l - 1] != y[l - 1]) reusable = 0;
+        if (!reusable) continue;
+        for (int t = 0; t < ntau; t++)
+          if (r[i - 1] <= tau[t]) num[t * np + u] += 1;
+      }
+    }
+  }
+}

@@ -50,6 +50,8 @@ def _bind(lib: ctypes.CDLL) -> ctypes.CDLL:
                                   vp, vp, vp, vp, vp, vp]
     lib.oracle_select.restype = i32
     lib.oracle_select.argtypes = [i32, i32, vp, vp, vp, vp, vp, f32, i32, i32, vp, vp, vp, vp]
+    lib.oracle_opportunity.restype = None
+    lib.oracle_opportunity.argtypes = [vp, vp, vp, vp, i32, i32, vp, i32, vp, i32, vp, vp]
     lib.oracle_lmhead_logits.restype = None
     lib.oracle_lmhead_logits.argtypes = [vp, vp, i32, i32, vp, i32, vp, vp]
     return lib
@@ -198,3 +200,21 @@ def lmhead_logits(h, W, tokens=None, lib: ctypes.CDLL | None = None) -> tuple[np
     out32 = np.zeros((T, V), np.float32)
     lib.oracle_lmhead_logits(_ptr(hb), _ptr(wb), H, V, _ptr(tok), T, _ptr(out64), _ptr(out32))
     return out64, out32
+
+
+def opportunity(row_argmax, draft, row_regret, taus, ps, status=None, lib: ctypes.CDLL | None = None):
+    """Eq. 4 counts: (num [len(taus), len(ps)] int64, den int) over the given blocks."""
+    lib = lib or load_library()
+    y = np.ascontiguousarray(row_argmax, dtype=np.int32)
+    n, K1 = y.shape
+    K = K1 - 1
+    x = np.ascontiguousarray(draft, dtype=np.int32).reshape(n, K)
+    r = np.ascontiguousarray(row_regret, dtype=np.float32).reshape(n, K)
+    st = None if status is None else np.ascontiguousarray(status, dtype=np.int32).reshape(n)
+    tau = np.ascontiguousarray(taus, dtype=np.float32)
+    p = np.ascontiguousarray(ps, dtype=np.int32)
+    num = np.zeros(len(tau) * len(p), np.int64)
+    den = np.zeros(1, np.int64)
+    lib.oracle_opportunity(_ptr(y), _ptr(x), _ptr(r), None if st is None else _ptr(st), n, K, _ptr(tau),
+                           len(tau), _ptr(p), len(p), _ptr(num), _ptr(den))
+    return num.reshape(len(tau), len(p)), int(den[0])

@@ -337,9 +337,37 @@ def pin_select_replays_verify(lib):
             assert np.array_equal(full[key], sel[key]), key
 
 
+def pin_opportunity_eq4(lib):
+    """Eq. 4 by explicit enumeration of the mismatch set M, and the Fig. 1 block by hand."""
+    rng = np.random.default_rng(19)
+    n, K = 200, 9
+    y = rng.integers(0, 4, size=(n, K + 1)).astype(np.int32)
+    x = y[:, :K].copy()
+    flip = rng.random((n, K)) < 0.35
+    x[flip] = (x[flip] + 1 + rng.integers(0, 3, size=flip.sum())) % 7
+    r = rng.choice(np.array([0.0, 0.25, 0.5, 1.0, 3.0], np.float32), size=(n, K))
+    status = (rng.random(n) < 0.1).astype(np.int32)
+    taus, ps = [0.0, 0.5, 1.0, float("inf")], [0, 1, 2, 3, 9]
+    num, den = oracle.opportunity(y, x, r, taus, ps, status=status, lib=lib)
+    M = [(b, i) for b in range(n) if status[b] == 0 for i in range(1, K + 1) if x[b, i - 1] != y[b, i - 1]]
+    assert den == len(M), "|M| is the number of mismatch positions"
+    for ti, tau in enumerate(taus):
+        for pi, pp in enumerate(ps):
+            expect = sum(1 for (b, i) in M if r[b, i - 1] <= tau and i + pp <= K
+                         and all(x[b, l - 1] == y[b, l - 1] for l in range(i + 1, i + pp + 1)))
+            assert num[ti, pi] == expect, f"Eq. 4 count (tau={tau}, p={pp})"
+    # Fig. 1 (K=4): one mismatch E (r = 0.5) at i = 1, then F and G match, X mismatches at i = 4
+    yf = np.array([[1, 3, 4, 5, 7]], np.int32)
+    xf = np.array([[2, 3, 4, 6]], np.int32)
+    rf = np.array([[0.5, 0.0, 0.0, 3.0]], np.float32)
+    num, den = oracle.opportunity(yf, xf, rf, [0.25, 1.0], [2, 3], lib=lib)
+    assert den == 2
+    assert num.tolist() == [[0, 0], [1, 0]], "E reuses F, G (p = 2) but not a third token"
+
+
 ALL_PINS = [pin_argmax_vs_numpy, pin_regret_vs_gather, pin_selection_bruteforce, pin_zero_budget_is_strict,
             pin_gate_and_budget_boundaries, pin_fig1, pin_cap_zero_is_strict, pin_carry_ledger,
-            pin_status_flags, pin_lmhead_vs_numpy, pin_select_replays_verify]
+            pin_status_flags, pin_lmhead_vs_numpy, pin_select_replays_verify, pin_opportunity_eq4]
 
 
 def run_all(lib, quick=False):

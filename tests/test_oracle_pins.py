@@ -59,6 +59,10 @@ def test_select_replays_verify(oracle_lib):
     P.pin_select_replays_verify(oracle_lib)
 
 
+def test_opportunity_statistic_eq4(oracle_lib):
+    P.pin_opportunity_eq4(oracle_lib)
+
+
 def test_k_zero_emits_bonus_only(oracle_lib):
     """K = 0 (no draft tokens): a = 0 = K, and the only emitted token is the bonus y*_1."""
     z = np.zeros((3, 1, 5), np.float32)
@@ -165,6 +169,9 @@ MUTANTS = {
     "strict stops one late": ("if (x[j] != y[j]) return j;", "if (x[j] != y[j]) return j + 1;"),
     "lm-head accumulates in fp32": ("double acc = 0.0;", "float acc = 0.0f;"),
     "lm-head ignores the token list": ("h + (int64_t)tokens[t] * H;", "h + (int64_t)t * H;"),
+    "opportunity counts the block end": ("int reusable = i + p[u] <= K;", "int reusable = i + p[u] <= K + 1;"),
+    "opportunity strict tau": ("if (r[i - 1] <= tau[t]) num[t * np + u] += 1;", "if (r[i - 1] < tau[t]) num[t * np + u] += 1;"),
+    "opportunity suffix starts at i": ("for (int l = i + 1; reusable && l <= i + p[u]; l++)", "for (int l = i; reusable && l < i + p[u]; l++)"),
 }
 
 
