@@ -218,6 +218,23 @@ int asd_verify_blocks(const void* logits, int dtype, int nblk, int B, int K, int
                       int32_t* row_argmax, float* row_regret, int32_t* status, void* workspace,
                       size_t workspace_bytes, asd_stream_t stream);
 
+/*
+ * The verifier-side opportunity rate of Eq. 4 (Sec. 3.1), as counts added to
+ * `counts` (device, uint64, accumulated over calls; zero it to start):
+ *   counts[t * np + u] += #{ mismatch positions (x, i) with r_i <= tau[t],
+ *                            i + p[u] <= K and x_l = y*_l for l = i+1 .. i+p[u] }
+ *   counts[ntau * np]  += |M|, the number of mismatch positions
+ * so Omega(tau[t], p[u]) = counts[t * np + u] / counts[ntau * np].
+ * row_argmax [n, K+1], draft [n, K], row_regret [n, K]: asd_verify's row
+ * outputs for n block-requests (device); status [n] or NULL (block-requests
+ * with a non-zero status are skipped). tau [ntau] and p [np] are HOST arrays,
+ * 1 <= ntau, np <= ASD_OPPORTUNITY_MAX; tau not NaN, p >= 0.
+ */
+#define ASD_OPPORTUNITY_MAX 16
+int asd_opportunity(const int32_t* row_argmax, const int32_t* draft, const float* row_regret,
+                    const int32_t* status, int n, int K, const float* tau, int ntau, const int32_t* p,
+                    int np, unsigned long long* counts, asd_stream_t stream);
+
 /* Human-readable text of a return code. Never NULL. */
 const char* asd_status_string(int code);
 

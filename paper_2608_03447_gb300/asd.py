@@ -62,6 +62,8 @@ def _declare(lib: ctypes.CDLL) -> ctypes.CDLL:
     lib.asd_verify_blocks.argtypes = [vp, i32, i32, i32, i32, i32, vp, vp, f32, i32, vp, vp, vp, vp, vp, vp, vp, sz,
                                       vp]
     lib.asd_verify_blocks.restype = i32
+    lib.asd_opportunity.argtypes = [vp, vp, vp, vp, i32, i32, vp, i32, vp, i32, vp, vp]
+    lib.asd_opportunity.restype = i32
     if hasattr(lib, "asd_verify_noalloc"):
         lib.asd_verify_noalloc.argtypes = [vp, i32, i32, i32, i32, vp, vp, f32, i32, vp, vp, vp, vp, vp, vp, vp]
         lib.asd_verify_noalloc.restype = i32
@@ -331,3 +333,21 @@ def verify_blocks(logits: torch.Tensor, draft: torch.Tensor, ledger: torch.Tenso
                                   ws.ptr, ws.nbytes, _stream(stream))
     _check("asd_verify_blocks", rc)
     return out
+
+
+def opportunity(row_argmax: torch.Tensor, draft: torch.Tensor, row_regret: torch.Tensor, taus, ps,
+                status: torch.Tensor | None = None, counts: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """asd_opportunity: Eq. 4 counts over the block-requests' row outputs (accumulated into ``counts``).
+
+    Returns the int64 counts tensor [len(taus) * len(ps) + 1] (the last entry is |M|).
+    """
+    import numpy as _np
+    n, K1 = row_argmax.shape[0], row_argmax.shape[-1]
+    tau = _np.ascontiguousarray(taus, dtype=_np.float32)
+    pv = _np.ascontiguousarray(ps, dtype=_np.int32)
+    if counts is None:
+        counts = torch.zeros(len(tau) * len(pv) + 1, dtype=torch.int64, device=row_argmax.device)
+    rc = load().asd_opportunity(_ptr(row_argmax), _ptr(draft), _ptr(row_regret), _ptr(status), n, K1 - 1,
+                                tau.ctypes.data, len(tau), pv.ctypes.data, len(pv), _ptr(counts), _stream(stream))
+    _check("asd_opportunity", rc)
+    return counts

@@ -1,0 +1,95 @@
+// libasd: the verifier-side opportunity rate of Eq. 4 (Sec. 3.1), as counts.
+//
+// Over every draft-target mismatch position (x, i) of the given blocks, count
+// those whose regret is at most tau and that are followed, inside the block,
+// by p draft tokens equal to the target's argmax; also count |M|. One thread
+// per block-request works on bit masks of the K positions: m (x_j == y*_j),
+// d = ~m, R_t (r_j <= tau_t) and S_p = AND_{k=1..p} (m >> k) (the next p
+// tokens match; bits past the block are zero, which also enforces i + p <= K),
+// then counts with popc. A CTA sums its threads in shared memory and adds to
+// the caller's counters once per counter.
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "asd.h"
+
+namespace {
+
+struct OpportunityArgs {
+  float tau[ASD_OPPORTUNITY_MAX];
+  int p[ASD_OPPORTUNITY_MAX];
+  int ntau, np;
+};
+
+constexpr int kStatThreads = 256;
+
+__global__ void __launch_bounds__(kStatThreads) opportunity_kernel(const int32_t* __restrict__ row_argmax,
+                                                                   const int32_t* __restrict__ draft,
+                                                                   const float* __restrict__ row_regret,
+                                                                   const int32_t* __restrict__ status, int n, int K,
+                                                                   const OpportunityArgs a,
+                                                                   unsigned long long* counts) {
+  __shared__ unsigned int local[ASD_OPPORTUNITY_MAX * ASD_OPPORTUNITY_MAX + 1];
+  const int ncount = a.ntau * a.np;
+  for (int i = threadIdx.x; i <= ncount; i += blockDim.x) local[i] = 0u;
+  __syncthreads();
+
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b < n && !(status && status[b] != 0)) {
+    const int32_t* y = row_argmax + static_cast<long long>(b) * (K + 1);
+    const int32_t* x = draft + static_cast<long long>(b) * K;
+    const float* r = row_regret + static_cast<long long>(b) * K;
+    uint32_t m = 0;
+    uint32_t rmask[ASD_OPPORTUNITY_MAX];
+    for (int t = 0; t < a.ntau; ++t) rmask[t] = 0u;
+    for (int j = 0; j < K; ++j) {
+      if (x[j] == y[j]) m |= 1u << j;
+      const float rj = r[j];
+      for (int t = 0; t < a.ntau; ++t)
+        if (rj <= a.tau[t]) rmask[t] |= 1u << j;
+    }
+    const uint32_t all = K >= 32 ? 0xffffffffu : ((1u << K) - 1u);
+    const uint32_t d = ~m & all;  // M restricted to this block
+    if (d) atomicAdd(&local[ncount], static_cast<unsigned>(__popc(d)));
+    for (int u = 0; u < a.np; ++u) {
+      uint32_t s = all;
+      for (int k = 1; k <= a.p[u] && s; ++k) s &= m >> k;
+      const uint32_t e = d & s;
+      if (!e) continue;
+      for (int t = 0; t < a.ntau; ++t) {
+        const int c = __popc(e & rmask[t]);
+        if (c) atomicAdd(&local[t * a.np + u], static_cast<unsigned>(c));
+      }
+    }
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i <= ncount; i += blockDim.x)
+    if (local[i]) atomicAdd(&counts[i], static_cast<unsigned long long>(local[i]));
+}
+
+}  // namespace
+
+extern "C" int asd_opportunity(const int32_t* row_argmax, const int32_t* draft, const float* row_regret,
+                               const int32_t* status, int n, int K, const float* tau, int ntau,
+                               const int32_t* p, int np, unsigned long long* counts, asd_stream_t stream) {
+  if (n < 0 || K < 0 || K > ASD_MAX_K) return ASD_ERR_SHAPE;
+  if (ntau < 1 || np < 1 || ntau > ASD_OPPORTUNITY_MAX || np > ASD_OPPORTUNITY_MAX) return ASD_ERR_SHAPE;
+  if (!tau || !p || !counts) return ASD_ERR_NULL;
+  OpportunityArgs a = {};
+  a.ntau = ntau;
+  a.np = np;
+  for (int t = 0; t < ntau; ++t) {
+    if (tau[t] != tau[t]) return ASD_ERR_CONTROL;
+    a.tau[t] = tau[t];
+  }
+  for (int u = 0; u < np; ++u) {
+    if (p[u] < 0) return ASD_ERR_CONTROL;
+    a.p[u] = p[u];
+  }
+  if (n == 0 || K == 0) return ASD_OK;  // no position can mismatch
+  if (!row_argmax || !draft || !row_regret) return ASD_ERR_NULL;
+  const unsigned grid = static_cast<unsigned>((n + kStatThreads - 1) / kStatThreads);
+  opportunity_kernel<<<grid, kStatThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
+      row_argmax, draft, row_regret, status, n, K, a, counts);
+  return cudaGetLastError() == cudaSuccess ? ASD_OK : ASD_ERR_CUDA;
+}
