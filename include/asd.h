@@ -46,6 +46,17 @@ typedef struct {
   float spent;
 } asd_ledger;
 
+/* One vocabulary shard's reduction of one target row (asd_shard_partials):
+ * what the tensor-parallel remark of Sec. 3.3 says the verifier needs from
+ * each shard, with no logit buffer. */
+typedef struct {
+  uint64_t key;        /* order-preserving (top logit, GLOBAL vocabulary index): larger wins */
+  float top;           /* the shard's top logit, exactly as stored (sign of zero kept) */
+  float draft_logit;   /* z(x) if the row's draft token is in this shard, else -INFINITY */
+  uint32_t flags;      /* ASD_STATUS_NAN_LOGIT if the shard saw a NaN in the row's request */
+  uint32_t reserved;
+} asd_partial;
+
 /* Logit storage types. */
 enum { ASD_F32 = 0, ASD_BF16 = 1 };
 
@@ -234,6 +245,28 @@ int asd_verify_blocks(const void* logits, int dtype, int nblk, int B, int K, int
 int asd_opportunity(const int32_t* row_argmax, const int32_t* draft, const float* row_regret,
                     const int32_t* status, int n, int K, const float* tau, int ntau, const int32_t* p,
                     int np, unsigned long long* counts, asd_stream_t stream);
+
+/*
+ * Vocabulary-sharded verify (Sec. 3.3: under tensor parallelism the verifier
+ * needs only the top token, the top logit and the draft token's logit, which
+ * each vocabulary shard can reduce locally). Step 1 on every shard:
+ *   asd_shard_partials: logits [B, K+1, Vs] hold the shard's vocabulary entries
+ *   v_offset .. v_offset+Vs-1 of a V-entry vocabulary; draft [B, K] holds
+ *   GLOBAL token ids; writes partials [B*(K+1)]. Workspace and its rules as for
+ *   asd_verify, sized with asd_workspace_size(B, K, Vs, dtype).
+ * Step 2, once the S shards' partials sit side by side (an all-gather across
+ * ranks, or S slices of one GPU):
+ *   asd_shard_combine: partials [S, B*(K+1)] -> the outputs of asd_verify for
+ *   the whole vocabulary, bit for bit (same keys, same fp32 arithmetic). No
+ *   workspace. The ledger, gate, cap and outputs are as in asd_verify.
+ */
+int asd_shard_partials(const void* logits, int dtype, int B, int K, int Vs, int v_offset, int V,
+                       const int32_t* draft, asd_partial* partials, void* workspace,
+                       size_t workspace_bytes, asd_stream_t stream);
+int asd_shard_combine(const asd_partial* partials, int S, int B, int K, int V, const int32_t* draft,
+                      asd_ledger* ledger, float gate, int cap, int32_t* accepted_len,
+                      int32_t* committed, int32_t* recovery, int32_t* row_argmax, float* row_regret,
+                      int32_t* status, asd_stream_t stream);
 
 /* Human-readable text of a return code. Never NULL. */
 const char* asd_status_string(int code);

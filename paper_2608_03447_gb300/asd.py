@@ -62,6 +62,10 @@ def _declare(lib: ctypes.CDLL) -> ctypes.CDLL:
     lib.asd_verify_blocks.argtypes = [vp, i32, i32, i32, i32, i32, vp, vp, f32, i32, vp, vp, vp, vp, vp, vp, vp, sz,
                                       vp]
     lib.asd_verify_blocks.restype = i32
+    lib.asd_shard_partials.argtypes = [vp, i32, i32, i32, i32, i32, i32, vp, vp, vp, sz, vp]
+    lib.asd_shard_partials.restype = i32
+    lib.asd_shard_combine.argtypes = [vp, i32, i32, i32, i32, vp, vp, f32, i32, vp, vp, vp, vp, vp, vp, vp]
+    lib.asd_shard_combine.restype = i32
     lib.asd_opportunity.argtypes = [vp, vp, vp, vp, i32, i32, vp, i32, vp, i32, vp, vp]
     lib.asd_opportunity.restype = i32
     if hasattr(lib, "asd_verify_noalloc"):
@@ -351,3 +355,47 @@ def opportunity(row_argmax: torch.Tensor, draft: torch.Tensor, row_regret: torch
                                 tau.ctypes.data, len(tau), pv.ctypes.data, len(pv), _ptr(counts), _stream(stream))
     _check("asd_opportunity", rc)
     return counts
+
+
+PARTIAL_WORDS = 6  # asd_partial: uint64 key, float top, float draft_logit, uint32 flags, uint32 reserved
+
+
+def shard_partials(logits: torch.Tensor, draft: torch.Tensor, v_offset: int, V: int,
+                   workspace: Workspace | None = None, out: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """asd_shard_partials: one vocabulary shard's per-row partials, as int32 [B*(K+1), 6] (asd_partial).
+
+    logits [B, K+1, Vs] hold vocabulary entries v_offset .. v_offset+Vs-1 of V; draft holds global ids.
+    """
+    B, K, Vs = _shape(logits, draft)
+    code = _dtype_code(logits)
+    ws = workspace or Workspace(B, K, Vs, code, logits.device, stream)
+    o = out if out is not None else torch.empty(B * (K + 1), PARTIAL_WORDS, dtype=torch.int32, device=logits.device)
+    rc = load().asd_shard_partials(_ptr(logits), code, B, K, Vs, int(v_offset), int(V), _ptr(draft), _ptr(o),
+                                   ws.ptr, ws.nbytes, _stream(stream))
+    _check("asd_shard_partials", rc)
+    return o
+
+
+def shard_combine(partials: torch.Tensor, draft: torch.Tensor, ledger: torch.Tensor, gate: float, cap: int, V: int,
+                  out: dict | None = None, stream=None) -> dict:
+    """asd_shard_combine: partials [S, B*(K+1), 6] of all shards -> the outputs of asd_verify."""
+    S, R, words = partials.shape
+    B, K = draft.shape
+    if words != PARTIAL_WORDS or R != B * (K + 1) or partials.dtype != torch.int32 or not partials.is_contiguous():
+        raise ValueError("partials must be a contiguous int32 tensor [S, B*(K+1), 6]")
+    o = out or alloc_outputs(B, K, partials.device)
+    rc = load().asd_shard_combine(_ptr(partials), S, B, K, int(V), _ptr(draft), _ptr(ledger), float(gate), int(cap),
+                                  _ptr(o["accepted_len"]), _ptr(o["committed"]), _ptr(o["recovery"]),
+                                  _ptr(o.get("row_argmax")), _ptr(o.get("row_regret")), _ptr(o.get("status")),
+                                  _stream(stream))
+    _check("asd_shard_combine", rc)
+    return o
+
+
+def allgather_partials(part: torch.Tensor, group=None) -> torch.Tensor:
+    """The exchange step of tensor-parallel verification: every rank's [B*(K+1), 6] partials -> [S, ...]."""
+    import torch.distributed as dist
+    world = dist.get_world_size(group)
+    parts = [torch.empty_like(part) for _ in range(world)]
+    dist.all_gather(parts, part.contiguous(), group=group)
+    return torch.stack(parts).contiguous()

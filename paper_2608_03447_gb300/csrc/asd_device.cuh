@@ -37,6 +37,9 @@ struct VerifyParams {
   unsigned int* error;          // sticky: ASD_ERR_TIMEOUT when a pipeline wait gave up
   float* row_top;               // [B*(K+1)] z_j(y*_j), or NULL (written by the fused LM-head path)
   int nblk;                     // sequential blocks of the same B requests (block i = requests i*B ..)
+  int v_offset;                 // vocabulary shard: global index of this shard's entry 0 (else 0)
+  int v_total;                  // vocabulary shard: entries of the whole vocabulary (else V)
+  asd_partial* partials;        // vocabulary shard: [B*(K+1)] outputs instead of the selection
 };
 
 // ---------------------------------------------------------------- element access
@@ -111,6 +114,8 @@ struct BlockInputs {
   int x;                   // draft token j (lanes < K)
   float zx;                // z_j(x_j) (lanes < K)
   unsigned flags;          // the block's status bits (every lane)
+  float top;               // z_j(y*_j) as the key holds it (a zero may have lost its sign)
+  bool top_exact;          // top is the stored value itself (sign of zero included)
 };
 
 __device__ __forceinline__ BlockInputs load_block(const VerifyParams& p, long long vb, int lane) {
@@ -135,6 +140,8 @@ __device__ __forceinline__ BlockInputs load_block(const VerifyParams& p, long lo
     p.flags[vb] = 0u;
   }
   in.flags = __shfl_sync(kFull, in.flags, 0);
+  in.top = ordered_value(static_cast<uint32_t>(in.key >> 32));
+  in.top_exact = false;
   return in;
 }
 
@@ -157,12 +164,12 @@ __device__ __forceinline__ void select_block(const VerifyParams& p, long long vb
   // Eq. 3: r_j = z_j(y*_j) - z_j(x_j). The key holds the maximum exactly, except
   // that it folds -0 onto +0; a zero maximum is re-read to keep its sign (when
   // the logits are in memory: the fused LM-head path passes none).
-  const float top = ordered_value(static_cast<uint32_t>(in.key >> 32));
+  const float top = in.top;
   float r = 0.0f;
   if (lane < K) {
     if (valid_x) {
       float t = top;
-      if (t == 0.0f && z) t = Elem<T>::load(z, row * p.V + y);
+      if (t == 0.0f && !in.top_exact && z) t = Elem<T>::load(z, row * p.V + y);
       r = __fsub_rn(t, in.zx);
     } else {
       r = __int_as_float(0x7fc00000);
@@ -219,8 +226,38 @@ __device__ __forceinline__ void select_block(const VerifyParams& p, long long vb
 // The selection of request b over its p.nblk blocks in order (block i is the
 // virtual request i * B + b): the ledger is read once, carried in registers
 // from block to block, and written once. Runs in one warp.
+// Vocabulary-shard mode: instead of selecting, hand each row's reduction of
+// this shard to the combine step (global index, exact top, draft logit).
+template <typename T>
+__device__ void emit_partials(const VerifyParams& p, int b, int lane) {
+  const int K = p.K, K1 = p.K + 1;
+  const T* z = static_cast<const T*>(p.logits);
+  BlockInputs in = load_block(p, b, lane);
+  if (lane < K1) {
+    const long long row = static_cast<long long>(b) * K1 + lane;
+    const uint32_t local = 0xffffffffu - static_cast<uint32_t>(in.key);
+    float top = in.top;
+    if (top == 0.0f && in.key) top = Elem<T>::load(z, row * p.V + local);  // keep the sign of a zero
+    const int xl = lane < K ? in.x - p.v_offset : -1;
+    asd_partial out;
+    out.key = in.key ? ((in.key & 0xffffffff00000000ull) |
+                        (0xffffffffu - (local + static_cast<uint32_t>(p.v_offset))))
+                     : 0ull;
+    out.top = top;
+    out.draft_logit = (xl >= 0 && xl < p.V) ? in.zx : -INFINITY;
+    out.flags = in.flags;
+    out.reserved = 0u;
+    p.partials[row] = out;
+  }
+  if (lane == 0) p.done[b] = 0ull;
+}
+
 template <typename T, bool kStrict>
 __device__ void select_request(const VerifyParams& p, int b, int lane) {
+  if (p.partials) {
+    emit_partials<T>(p, b, lane);
+    return;
+  }
   float budget = 0.0f, spent = 0.0f;
   if (!kStrict && lane == 0) {
     budget = p.ledger[b].budget;

@@ -202,7 +202,7 @@ __global__ void ASD_VERIFY_BOUNDS verify_kernel(const VerifyParams p) {
     const int b = static_cast<int>(row / K1);
     const int j = static_cast<int>(row - static_cast<long long>(b) * K1);
     int x = -1;
-    if (j < K) x = __ldg(p.draft + static_cast<long long>(b) * K + j);  // issued before the stream
+    if (j < K) x = __ldg(p.draft + static_cast<long long>(b) * K + j) - p.v_offset;  // shard-local
 
     if (b != pending_b) {  // finished this warp's share of block-request pending_b
       bool last = false;
@@ -385,7 +385,7 @@ __device__ __forceinline__ int draft_of_row(const VerifyParams& p, long long row
   const long long b = row / K1;
   const int j = static_cast<int>(row - b * K1);
   if (j >= p.K || b >= static_cast<long long>(p.B) * p.nblk) return -1;  // b: block-request
-  return __ldg(p.draft + b * p.K + j);
+  return __ldg(p.draft + b * p.K + j) - p.v_offset;  // shard-local (no shift without a shard)
 }
 
 __device__ __forceinline__ void cursor_enter(RowCursor& c, const VerifyParams& p, long long row) {
@@ -852,14 +852,16 @@ int verify_common(bool strict, const void* logits, int dtype, int B, int K, int 
                   const int32_t* draft, asd_ledger* ledger, float gate, int cap,
                   int32_t* accepted_len, int32_t* committed, int32_t* recovery,
                   int32_t* row_argmax, float* row_regret, int32_t* status, void* workspace,
-                  size_t workspace_bytes, cudaStream_t stream, int nblk = 1) {
+                  size_t workspace_bytes, cudaStream_t stream, int nblk = 1, int v_offset = 0,
+                  int v_total = 0, asd_partial* partials = nullptr) {
   int rc = check_shape(B, K, V, dtype);
   if (rc != ASD_OK) return rc;
   if (nblk < 0 || (nblk > 0 && B > INT32_MAX / nblk)) return ASD_ERR_SHAPE;
   if (B == 0 || nblk == 0) return ASD_OK;
-  if (!logits || !accepted_len || !committed || !recovery || !workspace) return ASD_ERR_NULL;
+  if (!logits || !workspace) return ASD_ERR_NULL;
+  if (!partials && (!accepted_len || !committed || !recovery)) return ASD_ERR_NULL;
   if (K > 0 && !draft) return ASD_ERR_NULL;
-  if (!strict) {
+  if (!strict && !partials) {
     if (!ledger) return ASD_ERR_NULL;
     if (gate != gate || gate < 0.0f || cap < 0) return ASD_ERR_CONTROL;
   }
@@ -874,6 +876,9 @@ int verify_common(bool strict, const void* logits, int dtype, int B, int K, int 
   p.K = K;
   p.V = V;
   p.nblk = nblk;
+  p.v_offset = v_offset;
+  p.v_total = v_total > 0 ? v_total : V;
+  p.partials = partials;
   p.total = static_cast<long long>(nblk) * B * (K + 1) * V;
   p.head = 0;
   p.per_warp = 0;
@@ -963,6 +968,16 @@ int asd_verify_blocks(const void* logits, int dtype, int nblk, int B, int K, int
   return verify_common(false, logits, dtype, B, K, V, draft, ledger, gate, cap, accepted_len, committed,
                        recovery, row_argmax, row_regret, status, workspace, workspace_bytes,
                        reinterpret_cast<cudaStream_t>(stream), nblk);
+}
+
+int asd_shard_partials(const void* logits, int dtype, int B, int K, int Vs, int v_offset, int V,
+                       const int32_t* draft, asd_partial* partials, void* workspace, size_t workspace_bytes,
+                       asd_stream_t stream) {
+  if (!partials) return ASD_ERR_NULL;
+  if (v_offset < 0 || Vs < 1 || V < 1 || static_cast<long long>(v_offset) + Vs > V) return ASD_ERR_SHAPE;
+  return verify_common(true, logits, dtype, B, K, Vs, draft, nullptr, 0.0f, 0, nullptr, nullptr, nullptr,
+                       nullptr, nullptr, nullptr, workspace, workspace_bytes,
+                       reinterpret_cast<cudaStream_t>(stream), 1, v_offset, V, partials);
 }
 
 const char* asd_status_string(int code) {

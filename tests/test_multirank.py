@@ -58,3 +58,64 @@ def test_single_rank_needs_no_process_group():
     import bench
     assert bench.max_over_ranks(3.5, "cpu", 1) == 3.5
     assert bench.job_rows_per_s(1, 288, 10, 0.5) == pytest.approx(5760.0)
+
+
+def _np_partials(z_shard, draft, v_offset):
+    """One shard's asd_partial rows (int32 [R, 6]) restated in numpy: the test's own key encoding."""
+    B, K1, Vs = z_shard.shape
+    K = K1 - 1
+    rows = z_shard.reshape(B * K1, Vs).astype(np.float32)
+    out = np.zeros((B * K1, 6), np.int32)
+    for r in range(B * K1):
+        loc = int(np.argmax(rows[r]))                    # first maximum
+        top = rows[r, loc]
+        u = np.array([top], np.float32).view(np.uint32)[0]
+        if (u << np.uint32(1)) == 0:
+            u = np.uint32(0)
+        o = (~u) if (u & 0x80000000) else (u | np.uint32(0x80000000))
+        key = (int(o) << 32) | (0xFFFFFFFF - (loc + v_offset))
+        out[r, 0:2] = np.array([key], np.uint64).view(np.int32)
+        out[r, 2] = np.array([top], np.float32).view(np.int32)[0]
+        b, j = divmod(r, K1)
+        zx = -np.inf
+        if j < K and v_offset <= draft[b, j] < v_offset + Vs:
+            zx = rows[r, draft[b, j] - v_offset]
+        out[r, 3] = np.array([zx], np.float32).view(np.int32)[0]
+    return out
+
+
+def _shard_rank(rank, world, port, result_dir):
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    sys.path.insert(0, root)
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank), WORLD_SIZE=str(world))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    from paper_2608_03447_gb300 import asd, inputs
+    blk = inputs.gen_block(3, 4, 999, torch.float32, 4242, "cpu")   # every rank generates the same block
+    V = blk.logits.shape[-1]
+    bounds = [0, 517, V]                                            # rank r holds vocabulary [bounds[r], bounds[r+1])
+    z = blk.logits.numpy()[:, :, bounds[rank]:bounds[rank + 1]]
+    part = torch.from_numpy(_np_partials(z, blk.draft.numpy(), bounds[rank]))
+    gathered = asd.allgather_partials(part)                        # the exchange step
+    np.save(os.path.join(result_dir, f"gathered{rank}.npy"), gathered.numpy())
+    dist.destroy_process_group()
+
+
+def test_two_gloo_ranks_exchange_vocab_partials(tmp_path):
+    from oracle import oracle
+    from paper_2608_03447_gb300 import inputs
+    world = 2
+    mp.spawn(_shard_rank, args=(world, _free_port(), str(tmp_path)), nprocs=world, join=True)
+    g0 = np.load(tmp_path / "gathered0.npy")
+    g1 = np.load(tmp_path / "gathered1.npy")
+    assert np.array_equal(g0, g1) and g0.shape[0] == 2              # every rank holds both shards' partials
+    keys = np.ascontiguousarray(g0[:, :, 0:2]).view(np.uint64)[..., 0]   # [S, R]
+    win = np.argmax(keys, axis=0)                                   # combine: the largest key
+    gidx = 0xFFFFFFFF - (keys[win, np.arange(keys.shape[1])] & 0xFFFFFFFF)
+    zx = np.where(g0[0, :, 3].view(np.float32) != -np.inf, g0[0, :, 3].view(np.float32), g0[1, :, 3].view(np.float32))
+    blk = inputs.gen_block(3, 4, 999, torch.float32, 4242, "cpu")
+    o = oracle.verify(blk.logits, blk.draft.numpy(), None, strict=True)
+    assert np.array_equal(gidx.reshape(3, 5), o["row_argmax"])
+    top = g0[win, np.arange(keys.shape[1]), 2].view(np.float32).reshape(3, 5)
+    r = (top[:, :4] - zx.reshape(3, 5)[:, :4]).astype(np.float32)
+    assert np.array_equal(r.view(np.uint32), o["row_regret"].view(np.uint32))
