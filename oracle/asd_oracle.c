@@ -288,3 +288,35 @@ void oracle_opportunity(const int32_t* row_argmax, const int32_t* draft, const f
     }
   }
 }
+
+/*
+ * Sec. 3.3, cache semantics: after a block is verified the caches and the
+ * history advance along the emitted sequence only. The emitted sequence of
+ * request b is committed[b][0..a] (x_1..x_a, then the recovery or bonus token).
+ *   tokens [B][max_tokens], token_len [B]: the history gets the a + 1 emitted
+ *     tokens appended at token_len[b]; token_len[b] += a + 1
+ *   kv_len [B]: the target cache keeps the pending input token (pending = 1 if
+ *     the verification pass consumed one before the drafts, else 0) and the a
+ *     accepted drafts: kv_len[b] += pending + a; positions from the new length
+ *     on held proposal-only state and are free
+ *   a request whose history has no room for a + 1 more tokens changes nothing
+ *     and gets status bit 8 (overflow)
+ * tokens / token_len / kv_len / status may be NULL (that part is skipped).
+ */
+void oracle_commit(int B, int K, const int32_t* accepted_len, const int32_t* committed, int pending,
+                   int32_t* kv_len, int32_t* tokens, int32_t* token_len, int max_tokens, int32_t* status) {
+  for (int b = 0; b < B; b++) {
+    int a = accepted_len[b];
+    const int32_t* emitted = committed + (int64_t)b * (K + 1);
+    if (tokens && token_len[b] + a + 1 > max_tokens) {
+      if (status) status[b] = 8;
+      continue;
+    }
+    if (status) status[b] = 0;
+    if (tokens) {
+      for (int j = 0; j <= a; j++) tokens[(int64_t)b * max_tokens + token_len[b] + j] = emitted[j];
+      token_len[b] += a + 1;
+    }
+    if (kv_len) kv_len[b] += pending + a;
+  }
+}

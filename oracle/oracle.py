@@ -52,6 +52,8 @@ def _bind(lib: ctypes.CDLL) -> ctypes.CDLL:
     lib.oracle_select.argtypes = [i32, i32, vp, vp, vp, vp, vp, f32, i32, i32, vp, vp, vp, vp]
     lib.oracle_opportunity.restype = None
     lib.oracle_opportunity.argtypes = [vp, vp, vp, vp, i32, i32, vp, i32, vp, i32, vp, vp]
+    lib.oracle_commit.restype = None
+    lib.oracle_commit.argtypes = [i32, i32, vp, vp, i32, vp, vp, vp, i32, vp]
     lib.oracle_lmhead_logits.restype = None
     lib.oracle_lmhead_logits.argtypes = [vp, vp, i32, i32, vp, i32, vp, vp]
     return lib
@@ -218,3 +220,17 @@ def opportunity(row_argmax, draft, row_regret, taus, ps, status=None, lib: ctype
     lib.oracle_opportunity(_ptr(y), _ptr(x), _ptr(r), None if st is None else _ptr(st), n, K, _ptr(tau),
                            len(tau), _ptr(p), len(p), _ptr(num), _ptr(den))
     return num.reshape(len(tau), len(p)), int(den[0])
+
+
+def commit(accepted_len, committed, pending, kv_len, tokens, token_len, lib: ctypes.CDLL | None = None) -> dict:
+    """Sec. 3.3 advance along the emitted sequence; returns updated copies (kv_len, tokens, token_len, status)."""
+    lib = lib or load_library()
+    a = np.ascontiguousarray(accepted_len, dtype=np.int32)
+    c = np.ascontiguousarray(committed, dtype=np.int32)
+    B, K1 = c.shape
+    kv = np.array(kv_len, dtype=np.int32, copy=True)
+    tok = np.array(tokens, dtype=np.int32, copy=True)
+    tl = np.array(token_len, dtype=np.int32, copy=True)
+    st = np.zeros(B, np.int32)
+    lib.oracle_commit(B, K1 - 1, _ptr(a), _ptr(c), int(pending), _ptr(kv), _ptr(tok), _ptr(tl), tok.shape[1], _ptr(st))
+    return {"kv_len": kv, "tokens": tok, "token_len": tl, "status": st}

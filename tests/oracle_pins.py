@@ -365,9 +365,26 @@ def pin_opportunity_eq4(lib):
     assert num.tolist() == [[0, 0], [1, 0]], "E reuses F, G (p = 2) but not a third token"
 
 
+def pin_commit_fig1(lib):
+    """Sec. 3.3 on the Fig. 1 case: E, F, G accepted, H emitted; the cache keeps the pending token and E, F, G."""
+    a = np.array([3, 0], np.int32)
+    committed = np.array([[2, 3, 4, 5, -1], [1, -1, -1, -1, -1]], np.int32)   # ASD and strict outputs
+    tokens = np.full((2, 8), -9, np.int32)
+    tokens[0, :2] = [10, 11]
+    res = oracle.commit(a, committed, 1, np.array([2, 5], np.int32), tokens, np.array([2, 0], np.int32), lib=lib)
+    assert res["tokens"][0].tolist() == [10, 11, 2, 3, 4, 5, -9, -9], "E F G H appended after the history"
+    assert res["tokens"][1].tolist() == [1, -9, -9, -9, -9, -9, -9, -9], "strict: only the recovery E'"
+    assert res["token_len"].tolist() == [6, 1]
+    assert res["kv_len"].tolist() == [2 + 1 + 3, 5 + 1 + 0]
+    full = oracle.commit(a, committed, 0, np.array([0, 0], np.int32), np.zeros((2, 4), np.int32),
+                         np.array([1, 4], np.int32), lib=lib)
+    assert full["status"].tolist() == [8, 8] and full["token_len"].tolist() == [1, 4], "no room: nothing changes"
+
+
 ALL_PINS = [pin_argmax_vs_numpy, pin_regret_vs_gather, pin_selection_bruteforce, pin_zero_budget_is_strict,
             pin_gate_and_budget_boundaries, pin_fig1, pin_cap_zero_is_strict, pin_carry_ledger,
-            pin_status_flags, pin_lmhead_vs_numpy, pin_select_replays_verify, pin_opportunity_eq4]
+            pin_status_flags, pin_lmhead_vs_numpy, pin_select_replays_verify, pin_opportunity_eq4,
+            pin_commit_fig1]
 
 
 def run_all(lib, quick=False):

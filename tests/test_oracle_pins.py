@@ -63,6 +63,10 @@ def test_opportunity_statistic_eq4(oracle_lib):
     P.pin_opportunity_eq4(oracle_lib)
 
 
+def test_commit_advances_along_the_emitted_sequence(oracle_lib):
+    P.pin_commit_fig1(oracle_lib)
+
+
 def test_k_zero_emits_bonus_only(oracle_lib):
     """K = 0 (no draft tokens): a = 0 = K, and the only emitted token is the bonus y*_1."""
     z = np.zeros((3, 1, 5), np.float32)
@@ -171,6 +175,8 @@ MUTANTS = {
     "lm-head ignores the token list": ("h + (int64_t)tokens[t] * H;", "h + (int64_t)t * H;"),
     "opportunity counts the block end": ("int reusable = i + p[u] <= K;", "int reusable = i + p[u] <= K + 1;"),
     "opportunity strict tau": ("if (r[i - 1] <= tau[t]) num[t * np + u] += 1;", "if (r[i - 1] < tau[t]) num[t * np + u] += 1;"),
+    "commit drops the recovery token": ("for (int j = 0; j <= a; j++) tokens", "for (int j = 0; j < a; j++) tokens"),
+    "commit forgets the pending token": ("if (kv_len) kv_len[b] += pending + a;", "if (kv_len) kv_len[b] += a;"),
     "opportunity suffix starts at i": ("for (int l = i + 1; reusable && l <= i + p[u]; l++)", "for (int l = i; reusable && l < i + p[u]; l++)"),
 }
 
