@@ -79,6 +79,7 @@ enum {
 #define ASD_STATUS_DRAFT_RANGE 1u /* a draft id outside [0, V) */
 #define ASD_STATUS_NAN_LOGIT 2u   /* a NaN among the request's K+1 logit rows */
 #define ASD_STATUS_BAD_LEDGER 4u  /* budget < 0 or NaN, spent < 0 or NaN, spent > budget */
+#define ASD_STATUS_OVERFLOW 8u    /* asd_commit: the token history has no room for the block */
 
 /* Largest draft length: one warp lane per target row of a block. */
 #define ASD_MAX_K 31
@@ -267,6 +268,27 @@ int asd_shard_combine(const asd_partial* partials, int S, int B, int K, int V, c
                       asd_ledger* ledger, float gate, int cap, int32_t* accepted_len,
                       int32_t* committed, int32_t* recovery, int32_t* row_argmax, float* row_regret,
                       int32_t* status, asd_stream_t stream);
+
+/*
+ * Advance along the emitted sequence (Sec. 3.3: the target cache, the draft
+ * cache and the ledger advance only along the emitted tokens; proposal-only
+ * state past the returned prefix is discarded). For each request b with
+ * a = accepted_len[b]:
+ *   tokens [B, max_tokens], token_len [B] (in/out): the a + 1 emitted tokens
+ *     committed[b][0..a] are appended at token_len[b]; token_len[b] += a + 1
+ *   kv_len [B] (in/out): kv_len[b] += pending + a -- the cache keeps the
+ *     pending input token of the pass (pending = 1 when the verification pass
+ *     consumed the previous round's recovery token before the drafts, else 0)
+ *     and the a accepted drafts; positions from the new length on held
+ *     proposal-only state and may be overwritten (call once per cache)
+ *   status [B] (out, may be NULL): ASD_STATUS_OVERFLOW when the history has
+ *     no room; such a request changes nothing.
+ * tokens / token_len may be NULL together, kv_len may be NULL. Device arrays.
+ * accepted_len values are those asd_verify writes (0..K); others are clamped.
+ */
+int asd_commit(int B, int K, const int32_t* accepted_len, const int32_t* committed, int pending,
+               int32_t* kv_len, int32_t* tokens, int32_t* token_len, int max_tokens, int32_t* status,
+               asd_stream_t stream);
 
 /* Human-readable text of a return code. Never NULL. */
 const char* asd_status_string(int code);

@@ -30,6 +30,7 @@ OK = 0
 STATUS_DRAFT_RANGE = 1
 STATUS_NAN_LOGIT = 2
 STATUS_BAD_LEDGER = 4
+STATUS_OVERFLOW = 8
 MAX_K = 31
 INT32_MAX = 2**31 - 1
 
@@ -66,6 +67,8 @@ def _declare(lib: ctypes.CDLL) -> ctypes.CDLL:
     lib.asd_shard_partials.restype = i32
     lib.asd_shard_combine.argtypes = [vp, i32, i32, i32, i32, vp, vp, f32, i32, vp, vp, vp, vp, vp, vp, vp]
     lib.asd_shard_combine.restype = i32
+    lib.asd_commit.argtypes = [i32, i32, vp, vp, i32, vp, vp, vp, i32, vp, vp]
+    lib.asd_commit.restype = i32
     lib.asd_opportunity.argtypes = [vp, vp, vp, vp, i32, i32, vp, i32, vp, i32, vp, vp]
     lib.asd_opportunity.restype = i32
     if hasattr(lib, "asd_verify_noalloc"):
@@ -399,3 +402,14 @@ def allgather_partials(part: torch.Tensor, group=None) -> torch.Tensor:
     parts = [torch.empty_like(part) for _ in range(world)]
     dist.all_gather(parts, part.contiguous(), group=group)
     return torch.stack(parts).contiguous()
+
+
+def commit(accepted_len: torch.Tensor, committed: torch.Tensor, pending: int = 1, kv_len: torch.Tensor | None = None,
+           tokens: torch.Tensor | None = None, token_len: torch.Tensor | None = None,
+           status: torch.Tensor | None = None, stream=None) -> None:
+    """asd_commit: append the emitted tokens to the history and advance the KV length (in place)."""
+    B, K1 = committed.shape
+    max_tokens = tokens.shape[1] if tokens is not None else 0
+    rc = load().asd_commit(B, K1 - 1, _ptr(accepted_len), _ptr(committed), int(pending), _ptr(kv_len), _ptr(tokens),
+                           _ptr(token_len), max_tokens, _ptr(status), _stream(stream))
+    _check("asd_commit", rc)

@@ -93,3 +93,51 @@ extern "C" int asd_opportunity(const int32_t* row_argmax, const int32_t* draft, 
       row_argmax, draft, row_regret, status, n, K, a, counts);
   return cudaGetLastError() == cudaSuccess ? ASD_OK : ASD_ERR_CUDA;
 }
+
+// ---------------------------------------------------------------- cache and history advance (Sec. 3.3)
+//
+// After a block is verified, the caches and the token history advance along
+// the emitted sequence only: committed[b][0..a]. One warp per request: lanes
+// 0..a append the emitted tokens to the history, lane 0 advances the lengths.
+
+namespace {
+
+constexpr int kCommitThreads = 256;
+
+__global__ void __launch_bounds__(kCommitThreads) commit_kernel(int B, int K, const int32_t* __restrict__ accepted_len,
+                                                                const int32_t* __restrict__ committed, int pending,
+                                                                int32_t* kv_len, int32_t* tokens, int32_t* token_len,
+                                                                int max_tokens, int32_t* status) {
+  const int lane = threadIdx.x & 31;
+  const int b = blockIdx.x * (kCommitThreads / 32) + (threadIdx.x >> 5);
+  if (b >= B) return;
+  int a = accepted_len[b];
+  a = a < 0 ? 0 : (a > K ? K : a);  // asd_verify writes 0..K; anything else is clamped (memory safety)
+  const int len = tokens ? token_len[b] : 0;
+  const bool room = !tokens || len + a + 1 <= max_tokens;
+  if (tokens && room && lane <= a)
+    tokens[static_cast<long long>(b) * max_tokens + len + lane] = committed[static_cast<long long>(b) * (K + 1) + lane];
+  if (lane == 0) {
+    if (status) status[b] = room ? 0 : ASD_STATUS_OVERFLOW;
+    if (room) {
+      if (tokens) token_len[b] = len + a + 1;
+      if (kv_len) kv_len[b] += pending + a;
+    }
+  }
+}
+
+}  // namespace
+
+extern "C" int asd_commit(int B, int K, const int32_t* accepted_len, const int32_t* committed, int pending,
+                          int32_t* kv_len, int32_t* tokens, int32_t* token_len, int max_tokens, int32_t* status,
+                          asd_stream_t stream) {
+  if (B < 0 || K < 0 || K > ASD_MAX_K || (pending != 0 && pending != 1)) return ASD_ERR_SHAPE;
+  if (B == 0) return ASD_OK;
+  if (!accepted_len || !committed) return ASD_ERR_NULL;
+  if (tokens && (!token_len || max_tokens < 1)) return ASD_ERR_NULL;
+  constexpr int kWarps = kCommitThreads / 32;
+  commit_kernel<<<static_cast<unsigned>((B + kWarps - 1) / kWarps), kCommitThreads, 0,
+                  reinterpret_cast<cudaStream_t>(stream)>>>(B, K, accepted_len, committed, pending, kv_len, tokens,
+                                                            token_len, max_tokens, status);
+  return cudaGetLastError() == cudaSuccess ? ASD_OK : ASD_ERR_CUDA;
+}
