@@ -245,27 +245,36 @@ __global__ void ASD_VERIFY_BOUNDS verify_kernel(const VerifyParams p) {
 
 // ---------------------------------------------------------------- TMA pipeline kernel
 //
-// One CTA per SM. The CTA owns an equal, 16-byte aligned slice of the flat
-// logits and streams it through a ring of shared-memory stages with bulk
-// copies (cp.async.bulk, completion counted on an mbarrier). A producer warp
-// keeps every free stage in flight, so the bytes in flight per SM are set by
-// the ring (kTmaStages x kTmaChunkBytes), not by registers. The consumer warps
-// each take a fixed sub-range of every chunk, so a warp visits its elements in
-// increasing order and keeps one running (value, index) per lane for the row
-// it is in; it flushes the row's key when it crosses into the next row, and
-// adds its element count to the request's counter when it crosses into the
-// next request (the last one to finish a request runs its selection).
+// One CTA per SM per launch. The CTA owns an equal, 16-byte aligned slice of
+// the flat logits and streams it through a ring of shared-memory stages with
+// bulk copies (cp.async.bulk, completion counted on an mbarrier). A producer
+// warp keeps every free stage in flight, so the bytes in flight per SM are set
+// by the ring, not by registers. Each consumer warp takes a fixed sub-range of
+// every chunk, so it visits its elements in increasing order and keeps one
+// running (value, index) per lane for the row it is in; finished rows merge
+// into a shared-memory row table (or straight into the workspace when a slice
+// spans more rows than the table holds). Nothing touches the workspace before
+// griddepcontrol.wait: every CTA signals its dependents at start, so the next
+// launches on the stream stream their own logits while this one ends. The
+// ring is small (4 x 16 KB) and registers are capped so that three CTAs --
+// three consecutive launches -- share an SM: one ramping up, one streaming, one
+// finishing. By default the selection then runs in select_kernel, launched
+// right behind (split mode); otherwise the CTAs count their elements per
+// request at the end and the last one to finish a request selects it.
 // Every wait is bounded (about a second of %globaltimer); on a timeout the CTA
 // records ASD_ERR_TIMEOUT in the workspace, stops, and drains its own copies.
 
 #ifndef ASD_TMA_STAGES
-#define ASD_TMA_STAGES 6  // 6 x 16 KB: two CTAs (this launch and the next) fit on one SM
+#define ASD_TMA_STAGES 4  // 4 x 16 KB: three CTAs (three consecutive launches) fit on one SM
 #endif
 #ifndef ASD_TMA_CHUNK_BYTES
 #define ASD_TMA_CHUNK_BYTES 16384
 #endif
 #ifndef ASD_TMA_CONSUMER_WARPS
 #define ASD_TMA_CONSUMER_WARPS 8
+#endif
+#ifndef ASD_TMA_MIN_BLOCKS
+#define ASD_TMA_MIN_BLOCKS 3  // CTAs per SM the register allocator must leave room for
 #endif
 #ifndef ASD_TMA_L2_HINT
 #define ASD_TMA_L2_HINT 1  // evict-first L2 policy on the streamed logits
@@ -544,8 +553,8 @@ __device__ __forceinline__ void consume_loose(RowCursor& c, const VerifyParams& 
   }
 }
 
-template <typename T, bool kStrict>
-__global__ void __launch_bounds__(kTmaThreads, 1)
+template <typename T, bool kStrict, bool kSplit>
+__global__ void __launch_bounds__(kTmaThreads, ASD_TMA_MIN_BLOCKS)
     verify_tma_kernel(const __grid_constant__ VerifyParams p, long long bulk_end, long long per_cta) {
   constexpr int VN = Elem<T>::kVec;
   constexpr int kChunkElems = kTmaChunkBytes / static_cast<int>(sizeof(T));
@@ -659,7 +668,8 @@ __global__ void __launch_bounds__(kTmaThreads, 1)
       consume_loose<T, kStrict>(c, p, sink, bulk_end, p.total, lane);
     }
     if (started && !sh.abort) cursor_flush_row<T>(c, p, sink, lane);
-    __threadfence();  // this warp's key merges and draft-logit stores, before the counts below
+    // this warp's direct key merges (slices spanning many rows) before the counts below
+    if (!kSplit && !sink.table) __threadfence();
   }
 
   __syncthreads();
@@ -688,9 +698,13 @@ __global__ void __launch_bounds__(kTmaThreads, 1)
       if (bits & 1u) atomicOr(&p.flags[row / (p.K + 1)], ASD_STATUS_NAN_LOGIT);
       if (bits & 2u) p.draft_logit[row] = sh.row_zx[t];
     }
+    // split mode: the selection runs in the next kernel, which the end of this
+    // grid orders after every write above; nothing more to do here
+    if (kSplit) return;
     __threadfence();
     __syncthreads();
   }
+  if (kSplit) return;
   if (cta_lo < cta_hi) {
     const long long rv = static_cast<long long>(p.K + 1) * p.V;
     const long long b_first = cta_lo / rv, b_last = (cta_hi - 1) / rv;
@@ -701,6 +715,27 @@ __global__ void __launch_bounds__(kTmaThreads, 1)
                                  static_cast<unsigned long long>(rv) * p.nblk, lane);
     }
   }
+}
+
+// ---------------------------------------------------------------- split selection kernel
+//
+// With the row stage in verify_tma_kernel<..., kSplit = true>, the selection of
+// every request runs here: one warp per request, launched right behind the row
+// stage (programmatic dependent launch); griddepcontrol.wait returns once the
+// row stage has completed and its writes are visible, so no counters and no
+// fences are needed, and the streaming CTAs leave their SMs as soon as they
+// have merged their rows.
+
+constexpr int kSelectThreads = 128;  // small: fits beside the streaming CTAs on an SM
+
+template <typename T, bool kStrict>
+__global__ void __launch_bounds__(kSelectThreads) select_kernel(const __grid_constant__ VerifyParams p) {
+  pdl_signal_dependents();
+  pdl_wait_prerequisites();
+  const int lane = threadIdx.x & 31;
+  const int warps = kSelectThreads / 32;
+  for (int b = blockIdx.x * warps + (threadIdx.x >> 5); b < p.B; b += gridDim.x * warps)
+    select_request<T, kStrict>(p, b, lane);
 }
 
 // ---------------------------------------------------------------- host side
@@ -737,8 +772,16 @@ int resident_warps(int* out) {
 
 struct DeviceInfo {
   int sms = 0;
-  bool tma_ready[4] = {false, false, false, false};
+  bool tma_ready[8] = {false, false, false, false, false, false, false, false};
 };
+
+// The TMA path's selection runs in its own kernel right behind the row stage
+// (see select_kernel); ASD_VERIFY_SPLIT=0 in the environment keeps it inside
+// the row-stage kernel instead (last-CTA-done), for comparison and testing.
+bool use_split() {
+  const char* env = getenv("ASD_VERIFY_SPLIT");
+  return !(env && env[0] == '0');
+}
 
 // SM count of the current device, and the one-time dynamic shared memory
 // opt-in of the TMA kernels, cached per device.
@@ -773,9 +816,11 @@ int launch_tma(VerifyParams& p, cudaStream_t stream) {
   DeviceInfo* info = nullptr;
   int rc = device_info(&dev, &info);
   if (rc != ASD_OK) return rc;
-  const int slot = (sizeof(T) == 2 ? 2 : 0) + (kStrict ? 1 : 0);
+  const bool split = use_split();
+  const int slot = (sizeof(T) == 2 ? 2 : 0) + (kStrict ? 1 : 0) + (split ? 4 : 0);
   if (!info->tma_ready[slot]) {
-    if (cudaFuncSetAttribute(verify_tma_kernel<T, kStrict>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    auto kernel = split ? verify_tma_kernel<T, kStrict, true> : verify_tma_kernel<T, kStrict, false>;
+    if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(sizeof(TmaShared))) != cudaSuccess)
       return ASD_ERR_CUDA;
     info->tma_ready[slot] = true;
@@ -803,8 +848,19 @@ int launch_tma(VerifyParams& p, cudaStream_t stream) {
     cfg.numAttrs = 1;
   }
   const long long bulk_end = head + bulk;
-  if (cudaLaunchKernelEx(&cfg, verify_tma_kernel<T, kStrict>, p, bulk_end, per_cta) != cudaSuccess)
+  if (!split) {
+    if (cudaLaunchKernelEx(&cfg, verify_tma_kernel<T, kStrict, false>, p, bulk_end, per_cta) != cudaSuccess)
+      return ASD_ERR_CUDA;
+    return cudaGetLastError() == cudaSuccess ? ASD_OK : ASD_ERR_CUDA;
+  }
+  if (cudaLaunchKernelEx(&cfg, verify_tma_kernel<T, kStrict, true>, p, bulk_end, per_cta) != cudaSuccess)
     return ASD_ERR_CUDA;
+  cudaLaunchConfig_t sel = cfg;
+  constexpr int kWarps = kSelectThreads / 32;
+  sel.gridDim = dim3(static_cast<unsigned>((p.B + kWarps - 1) / kWarps));
+  sel.blockDim = dim3(kSelectThreads);
+  sel.dynamicSmemBytes = 0;
+  if (cudaLaunchKernelEx(&sel, select_kernel<T, kStrict>, p) != cudaSuccess) return ASD_ERR_CUDA;
   return cudaGetLastError() == cudaSuccess ? ASD_OK : ASD_ERR_CUDA;
 }
 
