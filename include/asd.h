@@ -290,6 +290,11 @@ int asd_commit(int B, int K, const int32_t* accepted_len, const int32_t* committ
                int32_t* kv_len, int32_t* tokens, int32_t* token_len, int max_tokens, int32_t* status,
                asd_stream_t stream);
 
+/* How many kernels one asd_verify / asd_verify_strict call launches for this
+ * shape (1 or 2: the row stage, and for large inputs a separate selection
+ * kernel launched right behind it); 0 for B = 0. For accounting only. */
+int asd_verify_launches(int B, int K, int V, int dtype, int* launches);
+
 /* Human-readable text of a return code. Never NULL. */
 const char* asd_status_string(int code);
 

@@ -58,6 +58,8 @@ def _declare(lib: ctypes.CDLL) -> ctypes.CDLL:
     lib.asd_verify_strict.restype = i32
     lib.asd_status_string.argtypes = [i32]
     lib.asd_status_string.restype = ctypes.c_char_p
+    lib.asd_verify_launches.argtypes = [i32, i32, i32, i32, ctypes.POINTER(i32)]
+    lib.asd_verify_launches.restype = i32
     lib.asd_blocks_workspace_size.argtypes = [i32, i32, i32, i32, i32, ctypes.POINTER(sz)]
     lib.asd_blocks_workspace_size.restype = i32
     lib.asd_verify_blocks.argtypes = [vp, i32, i32, i32, i32, i32, vp, vp, f32, i32, vp, vp, vp, vp, vp, vp, vp, sz,
@@ -131,6 +133,13 @@ def _dtype_code(t: torch.Tensor) -> int:
     if t.dtype == torch.bfloat16:
         return BF16
     raise TypeError(f"logits must be float32 or bfloat16, got {t.dtype}")
+
+
+def verify_launches(B: int, K: int, V: int, dtype: int) -> int:
+    """asd_verify_launches: kernels one asd_verify call launches for this shape."""
+    n = ctypes.c_int(0)
+    _check("asd_verify_launches", load().asd_verify_launches(B, K, V, dtype, ctypes.byref(n)))
+    return n.value
 
 
 def workspace_size(B: int, K: int, V: int, dtype: int) -> int:

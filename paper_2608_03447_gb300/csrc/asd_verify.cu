@@ -1008,6 +1008,15 @@ int asd_verify_strict(const void* logits, int dtype, int B, int K, int V, const 
                        workspace_bytes, reinterpret_cast<cudaStream_t>(stream));
 }
 
+int asd_verify_launches(int B, int K, int V, int dtype, int* launches) {
+  if (!launches) return ASD_ERR_NULL;
+  const int rc = check_shape(B, K, V, dtype);
+  if (rc != ASD_OK) return rc;
+  const long long bytes = static_cast<long long>(B) * (K + 1) * V * (dtype == ASD_BF16 ? 2 : 4);
+  *launches = B == 0 ? 0 : (use_tma(bytes) && use_split() ? 2 : 1);
+  return ASD_OK;
+}
+
 int asd_blocks_workspace_size(int nblk, int B, int K, int V, int dtype, size_t* bytes) {
   if (!bytes) return ASD_ERR_NULL;
   const int rc = check_shape(B, K, V, dtype);
