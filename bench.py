@@ -342,6 +342,7 @@ def run_gpu(args) -> None:
     e2e = run_e2e(wl, dev, steps=max(10, min(steps, 200)), world=world)
 
     lm = run_lmhead(dev) if rank == 0 else None
+    nxt = run_next_rows(wl, dev) if rank == 0 else None
     if rank == 0:
         pk = peaks()
         cpu = cpu_baseline(wl) if world == 1 else None
@@ -365,6 +366,7 @@ def run_gpu(args) -> None:
             "gpu_launches": steps * asd.verify_launches(B, K, V, asd.BF16),
             "cpu_baseline": cpu,
             "fused_lmhead": lm,
+            "next_rows": nxt,
         }
         print(json.dumps(line), flush=True)
     if world > 1:
@@ -372,34 +374,140 @@ def run_gpu(args) -> None:
 
 
 def run_e2e(wl, dev, steps: int, world: int) -> dict:
-    """The same step through asd.verify_from_host: H2D of logits + drafts, verify, D2H of the results."""
+    """The same step through asd.verify_from_host: pinned host logits and drafts read in place by the
+    kernels over the host link, the per-request results copied back to pinned host memory."""
     from paper_2608_03447_gb300 import asd
     import torch.distributed as dist
     host_logits = [wl.logits[i].cpu().pin_memory() for i in range(2)]
     host_draft = [wl.drafts[i].cpu().pin_memory() for i in range(2)]
-    dev_logits = torch.empty_like(wl.logits[0])
-    dev_draft = torch.empty_like(wl.drafts[0])
     host_out = {k: torch.empty(v.shape, dtype=v.dtype, pin_memory=True)
                 for k, v in wl.out.items() if k in ("accepted_len", "committed", "recovery")}
     stream = torch.cuda.current_stream(dev)
     for i in range(3):
-        asd.verify_from_host(host_logits[i % 2], host_draft[i % 2], wl.ledger, GATE, CAP, dev_logits, dev_draft,
-                             wl.workspace, wl.out, host_out)
+        asd.verify_from_host(host_logits[i % 2], host_draft[i % 2], wl.ledger, GATE, CAP, wl.workspace, wl.out,
+                             host_out)
     torch.cuda.synchronize(dev)
     if world > 1:
         dist.barrier()
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     start.record(stream)
     for i in range(steps):
-        asd.verify_from_host(host_logits[i % 2], host_draft[i % 2], wl.ledger, GATE, CAP, dev_logits, dev_draft,
-                             wl.workspace, wl.out, host_out)
+        asd.verify_from_host(host_logits[i % 2], host_draft[i % 2], wl.ledger, GATE, CAP, wl.workspace, wl.out,
+                             host_out)
     end.record(stream)
     end.synchronize()
     sec = max_over_ranks(start.elapsed_time(end), dev, world) / 1e3
     h2d = host_logits[0].numel() * host_logits[0].element_size() + host_draft[0].numel() * 4
     d2h = sum(v.numel() * v.element_size() for v in host_out.values())
     return {"value": job_rows_per_s(world, B * (K + 1), steps, sec), "unit": "rows/s", "h2d_bytes_per_step": h2d,
-            "d2h_bytes_per_step": d2h, "steps": steps}
+            "d2h_bytes_per_step": d2h, "steps": steps, "host_link_gbs": h2d * steps / sec / 1e9,
+            "transfer": "kernels read the pinned host logits and drafts in place over the host link"}
+
+
+def _time(fn, dev, iters: int) -> float:
+    """Mean ms per call of fn over `iters` calls after 3 warm-up calls (CUDA events)."""
+    for _ in range(3):
+        fn()
+    torch.cuda.synchronize(dev)
+    stream = torch.cuda.current_stream(dev)
+    s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s.record(stream)
+    for _ in range(iters):
+        fn()
+    e.record(stream)
+    e.synchronize()
+    return s.elapsed_time(e) / iters
+
+
+def _time_graph(fn, dev, per_graph: int, replays: int = 5) -> float:
+    """Mean ms per call of fn, with `per_graph` calls captured in one CUDA graph (launch cost off the host)."""
+    fn()
+    torch.cuda.synchronize(dev)
+    side = torch.cuda.Stream(dev)
+    side.wait_stream(torch.cuda.current_stream(dev))
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=side):
+        for _ in range(per_graph):
+            fn()
+    for _ in range(2):
+        graph.replay()
+    torch.cuda.synchronize(dev)
+    stream = torch.cuda.current_stream(dev)
+    s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s.record(stream)
+    for _ in range(replays):
+        graph.replay()
+    e.record(stream)
+    e.synchronize()
+    return s.elapsed_time(e) / (replays * per_graph)
+
+
+def run_next_rows(wl, dev) -> dict:
+    """Throughput of the rows beyond the single-block step, on the same workload's buffers."""
+    from paper_2608_03447_gb300 import asd
+    pk = peaks()
+    out = {}
+    # multi-block: all rotating buffers as one call of nblk sequential blocks (> 4x L2 per call)
+    nblk = wl.nbuf
+    logits = torch.stack(wl.logits).contiguous()
+    drafts = torch.stack(wl.drafts).contiguous()
+    led = asd.make_ledger(B, BUDGET, 0.0, dev)
+    ws = asd.blocks_workspace(nblk, B, K, V, asd.BF16, dev)
+    flat = asd.alloc_outputs(nblk * B, K, dev)
+    res = {k: v.view(nblk, B, *v.shape[1:]) for k, v in flat.items()}
+    ms = _time(lambda: asd.verify_blocks(logits, drafts, led, GATE, CAP, ws, res), dev, 30)
+    gbs = logits.numel() * 2 / (ms * 1e-3) / 1e9
+    out["multi_block"] = {"workload": f"{nblk} sequential blocks of the step's batch per call", "ms_per_call": ms,
+                          "rows_per_s": nblk * B * (K + 1) / (ms * 1e-3), "hbm_gbs": gbs,
+                          "roofline": {"bound": "hbm", "achieved": gbs, "peak": pk["hbm_gbs"], "unit": "GB/s",
+                                       "frac": gbs / pk["hbm_gbs"]}}
+    del logits, drafts, flat, res
+    # vocabulary-sharded verify: 4 shards per block, partials then combine
+    S = 4
+    bounds = [round(V * i / S) for i in range(S + 1)]
+    shards = [[wl.logits[k][:, :, bounds[i]:bounds[i + 1]].contiguous() for i in range(S)] for k in range(wl.nbuf)]
+    parts = torch.empty(S, B * (K + 1), asd.PARTIAL_WORDS, dtype=torch.int32, device=dev)
+    sws = [asd.Workspace(B, K, bounds[i + 1] - bounds[i], asd.BF16, dev) for i in range(S)]
+    sled = asd.make_ledger(B, BUDGET, 0.0, dev)
+    sout = asd.alloc_outputs(B, K, dev)
+    step = [0]
+
+    def sharded():
+        k = step[0] % wl.nbuf
+        step[0] += 1
+        for i in range(S):
+            asd.shard_partials(shards[k][i], wl.drafts[k], bounds[i], V, sws[i], parts[i])
+        asd.shard_combine(parts, wl.drafts[k], sled, GATE, CAP, V, sout)
+
+    ms = _time_graph(sharded, dev, 4 * wl.nbuf)
+    gbs = B * (K + 1) * V * 2 / (ms * 1e-3) / 1e9
+    out["vocab_sharded"] = {"workload": f"{S} vocabulary shards per block (emulated tensor-parallel ranks), "
+                                        "partials + combine", "ms_per_step": ms,
+                            "rows_per_s": B * (K + 1) / (ms * 1e-3), "hbm_gbs": gbs,
+                            "roofline": {"bound": "hbm", "achieved": gbs, "peak": pk["hbm_gbs"], "unit": "GB/s",
+                                         "frac": gbs / pk["hbm_gbs"]}, "launches_per_step": S + 1}
+    del shards
+    # opportunity counts and history advance on the step's outputs (latency-bound, one launch each)
+    rows = asd.alloc_outputs(B, K, dev)
+    asd.verify(wl.logits[0], wl.drafts[0], asd.make_ledger(B, BUDGET, 0.0, dev), GATE, CAP, wl.workspace, rows)
+    counts = torch.zeros(4 * 4 + 1, dtype=torch.int64, device=dev)
+    ms = _time_graph(lambda: asd.opportunity(rows["row_argmax"], wl.drafts[0], rows["row_regret"],
+                                             [0.25, 0.5, 1.0, 2.0], [1, 2, 3, 4], counts=counts), dev, 100)
+    out["opportunity"] = {"workload": "Eq. 4 counts over the step's 32 x 8 positions, 4 taus x 4 ps",
+                          "us_per_call": ms * 1e3, "bound": "launch latency (graph of 100 calls)"}
+    tokens = torch.zeros(B, 4096, dtype=torch.int32, device=dev)
+    tlen = torch.zeros(B, dtype=torch.int32, device=dev)
+    kv = torch.zeros(B, dtype=torch.int32, device=dev)
+
+    def commit():
+        tlen.zero_()
+        asd.commit(rows["accepted_len"], rows["committed"], 1, kv, tokens, tlen)
+
+    ms = _time_graph(commit, dev, 100)
+    out["commit"] = {"workload": "append the step's emitted tokens and advance 32 KV lengths (with a zeroing of "
+                                 "the history length per call)", "us_per_call": ms * 1e3,
+                     "bound": "launch latency (graph of 100 calls)"}
+    return out
 
 
 def main():

@@ -290,6 +290,17 @@ int asd_commit(int B, int K, const int32_t* accepted_len, const int32_t* committ
                int32_t* kv_len, int32_t* tokens, int32_t* token_len, int max_tokens, int32_t* status,
                asd_stream_t stream);
 
+/* The device address through which kernels read page-locked (pinned) host
+ * memory, e.g. logits that stay in host memory and stream to the GPU over the
+ * host link while asd_verify runs, with no separate copy. `host` should lie in
+ * a pinned, mapped allocation (cudaHostAlloc / cudaHostRegister; runtime
+ * contexts map pinned memory by default). On systems whose GPU reads pageable
+ * memory through the host's page tables the runtime also accepts pageable
+ * memory (slower to read); where neither applies the call returns
+ * ASD_ERR_ALIGN. The alias is valid as long as the allocation is.
+ * Synchronous, no allocation. */
+int asd_host_alias(const void* host, void** device);
+
 /* How many kernels one asd_verify / asd_verify_strict call launches for this
  * shape (1 or 2: the row stage, and for large inputs a separate selection
  * kernel launched right behind it); 0 for B = 0. For accounting only. */

@@ -58,6 +58,8 @@ def _declare(lib: ctypes.CDLL) -> ctypes.CDLL:
     lib.asd_verify_strict.restype = i32
     lib.asd_status_string.argtypes = [i32]
     lib.asd_status_string.restype = ctypes.c_char_p
+    lib.asd_host_alias.argtypes = [vp, ctypes.POINTER(vp)]
+    lib.asd_host_alias.restype = i32
     lib.asd_verify_launches.argtypes = [i32, i32, i32, i32, ctypes.POINTER(i32)]
     lib.asd_verify_launches.restype = i32
     lib.asd_blocks_workspace_size.argtypes = [i32, i32, i32, i32, i32, ctypes.POINTER(sz)]
@@ -133,6 +135,15 @@ def _dtype_code(t: torch.Tensor) -> int:
     if t.dtype == torch.bfloat16:
         return BF16
     raise TypeError(f"logits must be float32 or bfloat16, got {t.dtype}")
+
+
+def host_alias(t: torch.Tensor) -> int:
+    """asd_host_alias: device address of a pinned host tensor's data (for reading it from kernels)."""
+    if t.is_cuda or not t.is_pinned():
+        raise ValueError("host_alias needs a pinned host tensor")
+    out = ctypes.c_void_p(0)
+    _check("asd_host_alias", load().asd_host_alias(t.data_ptr(), ctypes.byref(out)))
+    return out.value
 
 
 def verify_launches(B: int, K: int, V: int, dtype: int) -> int:
@@ -248,17 +259,36 @@ def verify_strict(logits: torch.Tensor, draft: torch.Tensor, workspace: Workspac
     return o
 
 
-def verify_from_host(logits_host: torch.Tensor, draft_host: torch.Tensor, ledger: torch.Tensor, gate: float,
-                     cap: int, logits_dev: torch.Tensor, draft_dev: torch.Tensor, workspace: Workspace,
-                     out: dict, host_out: dict, stream=None) -> dict:
-    """End-to-end step from pinned host buffers: copy in, verify, copy the per-request results out.
+_aliases: dict = {}
 
-    The ledger stays on the device (it is the request state carried between
-    rounds); the copies are asynchronous on ``stream``.
+
+def _alias(t: torch.Tensor) -> int:
+    key = (t.data_ptr(), t.numel() * t.element_size())
+    if key not in _aliases:
+        _aliases[key] = host_alias(t)
+    return _aliases[key]
+
+
+def verify_from_host(logits_host: torch.Tensor, draft_host: torch.Tensor, ledger: torch.Tensor, gate: float,
+                     cap: int, workspace: Workspace, out: dict, host_out: dict, stream=None) -> dict:
+    """End-to-end step from pinned host buffers: verify reading them in place, copy the results out.
+
+    The kernels read the pinned logits and drafts through their device aliases
+    (asd_host_alias), so the host-to-device transfer is the verify's own
+    stream of reads over the host link, with no separate copy; the ledger stays
+    on the device (the request state carried between rounds); the per-request
+    results are copied back to pinned host tensors, asynchronously on ``stream``.
     """
-    logits_dev.copy_(logits_host, non_blocking=True)
-    draft_dev.copy_(draft_host, non_blocking=True)
-    verify(logits_dev, draft_dev, ledger, gate, cap, workspace, out, stream)
+    if logits_host.dim() != 3 or not logits_host.is_pinned() or not draft_host.is_pinned():
+        raise ValueError("verify_from_host needs pinned host logits [B, K+1, V] and drafts [B, K]")
+    B, K1, V = logits_host.shape
+    K = K1 - 1
+    code = _dtype_code(logits_host)
+    rc = load().asd_verify(_alias(logits_host), code, B, K, V, _alias(draft_host), _ptr(ledger), float(gate),
+                           int(cap), _ptr(out["accepted_len"]), _ptr(out["committed"]), _ptr(out["recovery"]),
+                           _ptr(out.get("row_argmax")), _ptr(out.get("row_regret")), _ptr(out.get("status")),
+                           workspace.ptr, workspace.nbytes, _stream(stream))
+    _check("asd_verify", rc)
     for k in ("accepted_len", "committed", "recovery"):
         host_out[k].copy_(out[k], non_blocking=True)
     return host_out

@@ -1008,6 +1008,17 @@ int asd_verify_strict(const void* logits, int dtype, int B, int K, int V, const 
                        workspace_bytes, reinterpret_cast<cudaStream_t>(stream));
 }
 
+int asd_host_alias(const void* host, void** device) {
+  if (!host || !device) return ASD_ERR_NULL;
+  void* alias = nullptr;
+  if (cudaHostGetDevicePointer(&alias, const_cast<void*>(host), 0) != cudaSuccess || !alias) {
+    cudaGetLastError();  // clear the sticky-free error this query leaves behind
+    return ASD_ERR_ALIGN;
+  }
+  *device = alias;
+  return ASD_OK;
+}
+
 int asd_verify_launches(int B, int K, int V, int dtype, int* launches) {
   if (!launches) return ASD_ERR_NULL;
   const int rc = check_shape(B, K, V, dtype);

@@ -281,3 +281,29 @@ def test_full_size_graph_launch_matches_oracle(asd):
     g = _np(wl.out)
     g["ledger"] = wl.ledger.cpu().numpy()
     assert_parity(g, o, "graph replay, last step")
+
+
+def test_verify_reads_pinned_host_memory_in_place(asd, kernel):
+    """verify_from_host: kernels read pinned host logits through their device alias; same results."""
+    import ctypes
+
+    B, K, V = 8, 8, 70001
+    b = inputs.gen_block(B, K, V, torch.bfloat16, 5151, "cuda")
+    hl, hd = b.logits.cpu().pin_memory(), b.draft.cpu().pin_memory()
+    led_h, led_d = asd.make_ledger(B, 4.0), asd.make_ledger(B, 4.0)
+    ws = asd.Workspace(B, K, V, asd.BF16)
+    out = asd.alloc_outputs(B, K)
+    host_out = {k: torch.empty(out[k].shape, dtype=out[k].dtype, pin_memory=True)
+                for k in ("accepted_len", "committed", "recovery")}
+    for _ in range(2):  # two rounds: the ledger carries over
+        asd.verify_from_host(hl, hd, led_h, 1.0, 2, ws, out, host_out)
+        ref = asd.verify(b.logits, b.draft, led_d, 1.0, 2)
+        torch.cuda.synchronize()
+        for k in ("accepted_len", "committed", "recovery"):
+            assert torch.equal(host_out[k], ref[k].cpu()), k
+        assert torch.equal(out["row_argmax"], ref["row_argmax"])
+        assert torch.equal(led_h, led_d)
+    with pytest.raises(ValueError):
+        asd.host_alias(torch.zeros(4))  # the binding insists on pinned tensors
+    alias = ctypes.c_void_p(0)
+    assert asd.load().asd_host_alias(hl.data_ptr(), ctypes.byref(alias)) == 0 and alias.value
