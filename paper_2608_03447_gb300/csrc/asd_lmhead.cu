@@ -7,16 +7,23 @@
 // token's logit, with no [T, V] logit buffer); the selection of Alg. 1 then
 // runs as in asd_verify. The logits never reach global memory.
 //
-// Tiling: a CTA owns one 128-token tile (the MMA's M, TMEM lanes = tokens)
-// and loops over 256-wide vocabulary tiles (the MMA's N, TMEM columns), so each
-// epilogue thread owns one token and reduces its logits in registers. The grid
-// is (token tiles) x (CTAs per token tile); the CTAs that share a vocabulary
-// tile run at the same time, so each W tile comes from HBM once and from L2
-// for the other token tiles. Per CTA: warp 0 issues TMA loads (128B-swizzled
-// 64-wide K slabs) into a 4-stage ring, warp 1 allocates tensor memory and
-// issues tcgen05.mma from one thread, warps 2-5 read the accumulator with
-// tcgen05.ld; the 512 TMEM columns hold two 256-column accumulators so the
-// epilogue of one vocabulary tile overlaps the MMAs of the next.
+// Tiling: two CTAs on a pair of SMs (a cluster of 2) share one 2-SM MMA
+// (tcgen05 cta_group::2). The MMA's M is 256 vocabulary rows (128 per SM:
+// the TMEM lanes), its N is 192 token rows (the TMEM columns); each SM loads
+// its own 128 rows of W and half (96) of the token rows, so an SM takes in
+// 28 KB of operands per 64-deep K step for a 128 x 192 x 64 product, and the
+// 576 rows of a B = 64, K = 8 step are exactly three token tiles (no padded
+// rows). A pair owns one token tile and walks the vocabulary tiles with a
+// stride; the pairs of the three token tiles that share a vocabulary tile run
+// at the same time, so each W tile comes from HBM once and from L2 for the
+// other two. Per CTA: warp 0 issues TMA loads (128B-swizzled 64-wide K slabs)
+// into a kStages-deep ring, whose completion is counted on the first CTA's
+// barrier; warp 1 allocates tensor memory, and in the first CTA one of its
+// threads issues the MMAs; warps 2-5 read the accumulator with tcgen05.ld.
+// The 512 TMEM columns hold two 192-column accumulators, so the epilogue of
+// one vocabulary tile overlaps the MMAs of the next. The epilogue reduces
+// each token column over the 32 vocabulary rows of a warp with a transposing
+// butterfly of (value, index) keys and keeps a running key per token.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -32,29 +39,40 @@ namespace {
 
 using namespace asd_detail;
 
-constexpr int kBM = 128;                  // tokens per tile (MMA M)
-constexpr int kBN = 256;                  // vocabulary entries per tile (MMA N)
+constexpr int kPairM = 256;               // vocabulary rows per CTA pair (MMA M)
+constexpr int kHalfM = 128;               // vocabulary rows per CTA (TMEM lanes)
+constexpr int kTN = 192;                  // token rows per tile (MMA N)
+constexpr int kHalfN = kTN / 2;           // token rows each CTA of the pair loads
 constexpr int kBK = 64;                   // K per stage: 64 bf16 = one 128-byte swizzle row
 constexpr int kUmmaK = 16;                // K per tcgen05.mma (kind::f16)
-constexpr int kStages = 4;
-constexpr int kStageA = kBM * kBK * 2;    // 16 KB
-constexpr int kStageB = kBN * kBK * 2;    // 32 KB
+#ifndef ASD_LM_STAGES
+#define ASD_LM_STAGES 7
+#endif
+constexpr int kStages = ASD_LM_STAGES;
+constexpr int kStageB = kHalfN * kBK * 2;  // 12 KB of token rows
+constexpr int kStageA = kHalfM * kBK * 2;  // 16 KB of vocabulary rows
+constexpr uint32_t kStageTx = 2u * (kStageA + kStageB);  // both CTAs' bytes, counted on the first CTA
 constexpr int kLmThreads = 6 * 32;        // producer, MMA, 4 epilogue warps
-constexpr int kTmemCols = 2 * kBN;        // two accumulators
+constexpr int kTmemCols = 512;            // two accumulators at columns 0 and 256
+constexpr int kAccStride = 256;
+constexpr int kChunks = kTN / 32;         // 32-column TMEM loads per accumulator
+static_assert(kTN % 32 == 0 && kHalfN % 8 == 0, "token tile: whole 32-column loads, whole 8-row swizzle groups");
 
 struct LmShared {
-  unsigned long long full[kStages];
-  unsigned long long empty[kStages];
-  unsigned long long acc_full[2];
-  unsigned long long acc_empty[2];
+  unsigned long long full[kStages];   // first CTA: both CTAs' loads of a stage have landed
+  unsigned long long empty[kStages];  // each CTA: the MMAs have read its part of a stage
+  unsigned long long acc_full[2];     // each CTA: an accumulator is complete
+  unsigned long long acc_empty[2];    // first CTA: both CTAs' epilogues have read an accumulator
   unsigned long long drain;
   uint32_t tmem_base;
   int abort;
+  int draft[kTN];                     // x of the tile's token rows (-1: no draft / out of range)
 };
-// dynamic shared memory: [1 KB alignment slack][stages x (A, B)][LmShared]
+// dynamic shared memory: [1 KB alignment slack][stages x B][stages x A][LmShared]
 constexpr size_t kLmSmemBytes = 1024 + static_cast<size_t>(kStages) * (kStageA + kStageB) + sizeof(LmShared);
+static_assert(kLmSmemBytes <= 232448, "shared memory per CTA");
 
-// ---------------------------------------------------------------- tcgen05 / TMA helpers
+// ---------------------------------------------------------------- tcgen05 / TMA / cluster helpers
 
 // Shared-memory matrix descriptor of a K-major operand tile written by TMA with
 // 128-byte swizzling: rows of 128 bytes, 8-row groups 1024 bytes apart.
@@ -69,32 +87,85 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr) {
 }
 
 // Instruction descriptor: kind::f16 with bf16 A and B, fp32 D, both K-major,
-// M = kBM, N = kBN.
-constexpr uint32_t kIdesc = (1u << 4)                              // D format: f32
-                            | (1u << 7)                            // A format: bf16
-                            | (1u << 10)                           // B format: bf16
-                            | (static_cast<uint32_t>(kBN >> 3) << 17)  // N / 8
-                            | (static_cast<uint32_t>(kBM >> 4) << 24); // M / 16
+// M = kPairM (across the pair), N = kTN.
+constexpr uint32_t kIdesc = (1u << 4)                               // D format: f32
+                            | (1u << 7)                             // A format: bf16
+                            | (1u << 10)                            // B format: bf16
+                            | (static_cast<uint32_t>(kTN >> 3) << 17)     // N / 8
+                            | (static_cast<uint32_t>(kPairM >> 4) << 24); // M / 16
 
-__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, uint32_t bar, int x, int y) {
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// The shared::cluster address of the same shared-memory location in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t map_rank(uint32_t saddr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait_cluster(unsigned long long* bar, uint32_t parity) {
+  uint32_t done;
   asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];"
-      ::"r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(x), "r"(y)
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(done)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return done != 0;
+}
+// mbar_wait for barriers that the other CTA of the pair also signals.
+__device__ inline bool mbar_wait_cluster(unsigned long long* bar, uint32_t parity, volatile int* abort) {
+  if (mbar_try_wait_cluster(bar, parity)) return true;
+  const unsigned long long t0 = global_ns();
+  for (unsigned it = 1;; ++it) {
+    if (mbar_try_wait_cluster(bar, parity)) return true;
+    if ((it & 255u) == 0) {
+      if (*abort) return false;
+      if (global_ns() - t0 > kWaitLimitNs) return false;
+    }
+  }
+}
+
+// TMA tile load into this CTA's shared memory whose completion is counted on
+// an mbarrier of either CTA of the pair (cluster address).
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap* map, uint32_t bar_cluster, int x,
+                                                 int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.cta_group::2"
+      " [%0], [%1, {%3, %4}], [%2];"
+      ::"r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster), "r"(x), "r"(y)
       : "memory");
 }
 
-__device__ __forceinline__ void umma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t accumulate) {
+__device__ __forceinline__ void umma_pair_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t accumulate) {
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
       "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}"
       ::"r"(tmem_d), "l"(adesc), "l"(bdesc), "r"(kIdesc), "r"(accumulate)
       : "memory");
 }
 
-// The mbarrier arrives once every tcgen05 operation this thread issued so far has completed.
-__device__ __forceinline__ void umma_commit(unsigned long long* bar) {
-  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];"
+// The mbarrier at this offset in both CTAs of the pair arrives once every
+// tcgen05 operation this thread issued so far has completed.
+__device__ __forceinline__ void umma_commit_pair(unsigned long long* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;"
+      ::"r"(smem_u32(bar)), "h"(static_cast<uint16_t>(0x3)) : "memory");
+}
+// Same, for this CTA's barrier only.
+__device__ __forceinline__ void umma_commit_local(unsigned long long* bar) {
+  asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];"
                ::"r"(smem_u32(bar)) : "memory");
 }
 
@@ -124,17 +195,46 @@ __device__ __forceinline__ void report_timeout(const VerifyParams& p) {
   if (p.error) atomicExch(p.error, static_cast<unsigned>(ASD_ERR_TIMEOUT));
 }
 
+// Sets the abort flag of both CTAs of the pair.
+__device__ __forceinline__ void abort_pair(LmShared& sh, uint32_t peer) {
+  sh.abort = 1;
+  asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(map_rank(smem_u32(&sh.abort), peer)), "r"(1) : "memory");
+}
+
+// Order-preserving bits of a column maximum; NaN is mapped above +inf
+// whatever its sign bit, so a NaN anywhere in a row reaches the row's key.
+__device__ __forceinline__ uint32_t max_bits(float v) { return v != v ? 0xffc00000u : ordered_bits(v); }
+
+// Warp-wide transposing maximum: lane l holds the logits of its vocabulary
+// row for 32 token columns (z[0..31]); afterwards lane l holds, in z[0], the
+// maximum over the 32 lanes of column l (NaN if any of them is NaN). Five
+// exchange levels; at each the lane keeps the half of its columns selected
+// by its lane bit and receives the partner's values for that half.
+__device__ __forceinline__ float transpose_max32(float (&z)[32], int lane) {
+#pragma unroll
+  for (int half = 16; half >= 1; half >>= 1) {
+    const bool up = (lane & half) != 0;
+#pragma unroll
+    for (int i = 0; i < half; ++i) {
+      const float send = up ? z[i] : z[i + half];
+      const float keep = up ? z[i + half] : z[i];
+      z[i] = fmax_nan(keep, __shfl_xor_sync(kFull, send, half));
+    }
+  }
+  return z[0];
+}
+
 struct LmParams {
   int T, H, V;
-  int token_tiles;     // ceil(T / kBM)
-  int ctas_per_tile;   // CTAs that share one token tile
-  int vocab_tiles;     // ceil(V / kBN)
+  int token_tiles;     // ceil(T / kTN)
+  int pairs_per_tile;  // CTA pairs that share one token tile
+  int vocab_tiles;     // ceil(V / kPairM)
   int k_steps;         // ceil(H / kBK)
   float* logits_out;   // [T, V] when writing logits instead of verifying
 };
 
-// One CTA: token tile m = blockIdx.x % token_tiles, vocabulary tiles
-// n = blockIdx.x / token_tiles + i * ctas_per_tile.
+// One CTA pair (cluster of 2): token tile m = pair % token_tiles, vocabulary
+// tiles n = pair / token_tiles + i * pairs_per_tile.
 template <bool kStrict, bool kWriteLogits>
 __global__ void __launch_bounds__(kLmThreads, 1)
     lmhead_verify_kernel(const __grid_constant__ CUtensorMap map_h, const __grid_constant__ CUtensorMap map_w,
@@ -143,14 +243,20 @@ __global__ void __launch_bounds__(kLmThreads, 1)
   const uint32_t raw = smem_u32(lm_smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;  // 1024-byte aligned for the 128-byte swizzle
   unsigned char* gbase = lm_smem_raw + (base - raw);
-  const uint32_t sA = base;                                        // kStages x kStageA
-  const uint32_t sB = base + kStages * kStageA;                    // kStages x kStageB
+  const uint32_t sB = base;                                        // kStages x kStageB
+  const uint32_t sA = base + kStages * kStageB;                    // kStages x kStageA
   LmShared& sh = *reinterpret_cast<LmShared*>(gbase + kStages * (kStageA + kStageB));
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int m = static_cast<int>(blockIdx.x) % q.token_tiles;
-  const int n_first = static_cast<int>(blockIdx.x) / q.token_tiles;
-  const int n_tiles = n_first < q.vocab_tiles ? (q.vocab_tiles - n_first + q.ctas_per_tile - 1) / q.ctas_per_tile : 0;
+  const uint32_t rank = cluster_rank() & 1u;
+  const uint32_t peer = rank ^ 1u;
+  const bool leader = rank == 0;
+  const int pair = static_cast<int>(blockIdx.x >> 1);
+  const int m = pair % q.token_tiles;
+  const int n_first = pair / q.token_tiles;
+  const int n_tiles =
+      n_first < q.vocab_tiles ? (q.vocab_tiles - n_first + q.pairs_per_tile - 1) / q.pairs_per_tile : 0;
+  const int K1 = p.K + 1;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
@@ -159,63 +265,77 @@ __global__ void __launch_bounds__(kLmThreads, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&sh.acc_full[a], 1);
-      mbar_init(&sh.acc_empty[a], 4);
+      mbar_init(&sh.acc_empty[a], 8);  // 4 epilogue warps in each CTA
     }
     mbar_init(&sh.drain, 1);
     sh.abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
-  if (warp == 1) {  // tensor memory: 512 columns (this CTA is alone on its SM: see kLmSmemBytes)
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;"
+  if (!kWriteLogits) {
+    for (int c = threadIdx.x; c < kTN; c += kLmThreads) {
+      const int tok = m * kTN + c;
+      int x = -1;
+      if (tok < q.T && (tok % K1) < p.K) {
+        x = __ldg(p.draft + static_cast<long long>(tok / K1) * p.K + (tok % K1));
+        if (x < 0 || x >= p.V) x = -1;
+      }
+      sh.draft[c] = x;
+    }
+  }
+  if (warp == 1) {  // tensor memory of both SMs, allocated together by one warp of each CTA
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;"
                  ::"r"(smem_u32(&sh.tmem_base)), "r"(kTmemCols) : "memory");
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
   }
   tc_fence_before();
   __syncthreads();
+  cluster_sync_all();  // both CTAs' barriers exist before either signals the other's
   tc_fence_after();
   const uint32_t tmem = sh.tmem_base;
 
   int it_issued = 0;
   if (warp == 0) {
-    // ---------------- TMA producer
+    // ---------------- TMA producer (both CTAs; completion counted on the first CTA's barrier)
     if (lane == 0) {
       asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&map_h)) : "memory");
       asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&map_w)) : "memory");
+      const uint32_t full0 = map_rank(smem_u32(&sh.full[0]), 0);
       int it = 0;
       for (int t = 0; t < n_tiles && !sh.abort; ++t) {
-        const int n = n_first + t * q.ctas_per_tile;
+        const int n = n_first + t * q.pairs_per_tile;
         for (int k = 0; k < q.k_steps; ++k, ++it) {
           const int s = it % kStages;
-          if (!mbar_wait(&sh.empty[s], ((it / kStages) & 1) ^ 1, &sh.abort)) {
-            sh.abort = 1;
+          if (!mbar_wait_cluster(&sh.empty[s], ((it / kStages) & 1) ^ 1, &sh.abort)) {
+            abort_pair(sh, peer);
             report_timeout(p);
             break;
           }
-          mbar_expect_tx(&sh.full[s], kStageA + kStageB);
-          tma_load_2d(sA + s * kStageA, &map_h, smem_u32(&sh.full[s]), k * kBK, m * kBM);
-          tma_load_2d(sB + s * kStageB, &map_w, smem_u32(&sh.full[s]), k * kBK, n * kBN);
+          if (leader) mbar_expect_tx(&sh.full[s], kStageTx);
+          const uint32_t bar = full0 + static_cast<uint32_t>(s * sizeof(unsigned long long));
+          tma_load_2d_pair(sB + s * kStageB, &map_h, bar, k * kBK, m * kTN + static_cast<int>(rank) * kHalfN);
+          tma_load_2d_pair(sA + s * kStageA, &map_w, bar, k * kBK, n * kPairM + static_cast<int>(rank) * kHalfM);
           it_issued = it + 1;
         }
       }
     }
   } else if (warp == 1) {
-    // ---------------- MMA issuer (one thread)
-    if (lane == 0) {
+    // ---------------- MMA issuer (one thread of the first CTA, for both SMs)
+    if (leader && lane == 0) {
       int it = 0;
       for (int t = 0; t < n_tiles && !sh.abort; ++t) {
         const int a = t & 1;
-        if (!mbar_wait(&sh.acc_empty[a], ((t >> 1) & 1) ^ 1, &sh.abort)) {
-          sh.abort = 1;
+        if (!mbar_wait_cluster(&sh.acc_empty[a], ((t >> 1) & 1) ^ 1, &sh.abort)) {
+          abort_pair(sh, peer);
           report_timeout(p);
           break;
         }
         tc_fence_after();
-        const uint32_t d = tmem + static_cast<uint32_t>(a * kBN);
+        const uint32_t d = tmem + static_cast<uint32_t>(a * kAccStride);
         bool ok = true;
         for (int k = 0; k < q.k_steps; ++k, ++it) {
           const int s = it % kStages;
-          if (!mbar_wait(&sh.full[s], (it / kStages) & 1, &sh.abort)) {
+          if (!mbar_wait_cluster(&sh.full[s], (it / kStages) & 1, &sh.abort)) {
             ok = false;
             break;
           }
@@ -225,117 +345,150 @@ __global__ void __launch_bounds__(kLmThreads, 1)
 #pragma unroll
           for (int kk = 0; kk < kBK / kUmmaK; ++kk) {
             // advance 16 elements (32 bytes, encoded 2) along K inside the swizzle row
-            umma_bf16(d, ad + 2u * kk, bd + 2u * kk, (k > 0 || kk > 0) ? 1u : 0u);
+            umma_pair_bf16(d, ad + 2u * kk, bd + 2u * kk, (k > 0 || kk > 0) ? 1u : 0u);
           }
-          umma_commit(&sh.empty[s]);  // frees the stage when these MMAs have read it
+          umma_commit_pair(&sh.empty[s]);  // frees the stage in both CTAs when these MMAs have read it
         }
         if (!ok) {
-          sh.abort = 1;
+          abort_pair(sh, peer);
           report_timeout(p);
           break;
         }
-        umma_commit(&sh.acc_full[a]);  // the accumulator is complete
+        umma_commit_pair(&sh.acc_full[a]);  // the accumulator is complete in both CTAs
       }
-      umma_commit(&sh.drain);  // arrives once every MMA issued above has finished
+      umma_commit_local(&sh.drain);  // arrives once every MMA issued above has finished
       const unsigned long long t0 = global_ns();
       while (!mbar_try_wait(&sh.drain, 0) && global_ns() - t0 < kWaitLimitNs) {
       }
     }
   } else {
-    // ---------------- epilogue: warps 2-5, one token row per thread
+    // ---------------- epilogue: warps 2-5, one vocabulary row (TMEM lane) per thread
     const int quarter = warp & 3;                     // TMEM lanes this warp may read
-    const int row = quarter * 32 + lane;              // row of the token tile
-    const int tok = m * kBM + row;                    // global token row
-    const bool valid = tok < q.T;
-    const int K1 = p.K + 1;
-    int x = -1;
-    if (!kWriteLogits && valid && (tok % K1) < p.K) {
-      x = __ldg(p.draft + static_cast<long long>(tok / K1) * p.K + (tok % K1));
-      if (x < 0 || x >= p.V) x = -1;
-    }
-    float best = -INFINITY, zx = 0.0f, nan_acc = 0.0f;
-    int best_i = -1;
-    bool has_zx = false;
     const uint32_t lane_base = static_cast<uint32_t>(quarter * 32) << 16;
+    const uint32_t acc_empty0 = map_rank(smem_u32(&sh.acc_empty[0]), 0);
+    int xs[kChunks];  // lane l: draft of token column c * 32 + l
+#pragma unroll
+    for (int c = 0; c < kChunks; ++c) xs[c] = kWriteLogits ? -1 : sh.draft[c * 32 + lane];
+    unsigned long long best[kChunks];  // lane l: running key of token column c * 32 + l
+#pragma unroll
+    for (int c = 0; c < kChunks; ++c) best[c] = 0ull;
     for (int t = 0; t < n_tiles; ++t) {
       const int a = t & 1;
-      const bool ok = __all_sync(kFull, mbar_wait(&sh.acc_full[a], (t >> 1) & 1, &sh.abort));
+      const bool ok = __all_sync(kFull, mbar_wait_cluster(&sh.acc_full[a], (t >> 1) & 1, &sh.abort));
       if (!ok) {
-        sh.abort = 1;
-        if (lane == 0) report_timeout(p);
+        if (lane == 0) {
+          abort_pair(sh, peer);
+          report_timeout(p);
+        }
         break;
       }
       tc_fence_after();
-      const int n0 = (n_first + t * q.ctas_per_tile) * kBN;
-#pragma unroll 1
-      for (int c = 0; c < kBN; c += 32) {
+      const int v_warp = (n_first + t * q.pairs_per_tile) * kPairM + static_cast<int>(rank) * kHalfM + quarter * 32;
+      const int v = v_warp + lane;  // this thread's vocabulary row
+#pragma unroll
+      for (int c = 0; c < kChunks; ++c) {
         uint32_t r[32];
-        tmem_ld32(tmem + lane_base + static_cast<uint32_t>(a * kBN + c), r);
+        tmem_ld32(tmem + lane_base + static_cast<uint32_t>(a * kAccStride + c * 32), r);
         tmem_ld_wait();
         if (kWriteLogits) {
-          if (valid) {
-            float* out = q.logits_out + static_cast<long long>(tok) * q.V + n0 + c;
+          if (v < q.V) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i)
-              if (n0 + c + i < q.V) out[i] = __uint_as_float(r[i]);
+            for (int i = 0; i < 32; ++i) {
+              const int tok = m * kTN + c * 32 + i;
+              if (tok < q.T) q.logits_out[static_cast<long long>(tok) * q.V + v] = __uint_as_float(r[i]);
+            }
           }
         } else {
+          // draft logits: the lane holding row x of column i keeps z_i(x) (rare: at most one row per column)
+          unsigned hit = __ballot_sync(kFull, static_cast<unsigned>(xs[c] - v_warp) < 32u);
+          while (hit) {
+            const int i = __ffs(hit) - 1;
+            hit &= hit - 1;
+            const int owner = __shfl_sync(kFull, xs[c], i) - v_warp;
+            if (lane == owner) {
+              float z = 0.0f;
 #pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const int col = n0 + c + i;
-            const float v = __uint_as_float(r[i]);
-            if (col < q.V) {
-              nan_acc = fmax_nan(nan_acc, v);
-              if (v > best || best_i < 0) {  // columns arrive in increasing order: first maximum kept
-                best = v;
-                best_i = col;
+              for (int j = 0; j < 32; ++j)
+                if (j == i) z = __uint_as_float(r[j]);
+              p.draft_logit[m * kTN + c * 32 + i] = z;
+            }
+          }
+          // argmax of each column over the warp's 32 rows: the maximum by a
+          // transposing butterfly, then, for the columns whose running maximum
+          // it raises, the lowest row holding it (a ballot of equal values).
+          if (v_warp >= q.V) continue;  // rows past the vocabulary: nothing to reduce
+          float z[32];
+#pragma unroll
+          for (int i = 0; i < 32; ++i) z[i] = __uint_as_float(r[i]);
+          if (v_warp + 31 >= q.V) {  // the last, partial tile: rows past V never win
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+              if (v >= q.V) z[i] = -INFINITY;
+          }
+          const float zmax = transpose_max32(z, lane);
+          const uint32_t hi = max_bits(zmax);
+          const unsigned raise = __ballot_sync(kFull, hi > static_cast<uint32_t>(best[c] >> 32));
+          if (raise) {
+            unsigned rows = 0;  // lane l: rows of column l that hold its maximum
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              if ((raise >> i) & 1u) {
+                const float zi = __shfl_sync(kFull, zmax, i);
+                const float mine = v < q.V ? __uint_as_float(r[i]) : -INFINITY;
+                const unsigned eq = __ballot_sync(kFull, mine == zi);
+                if (lane == i) rows = eq;
               }
-              if (col == x) {
-                zx = v;
-                has_zx = true;
-              }
+            }
+            if ((raise >> lane) & 1u) {
+              const int w = rows ? __ffs(rows) - 1 : 0;  // NaN: no row compares equal; the key still says NaN
+              best[c] = (static_cast<unsigned long long>(hi) << 32) | (0xffffffffu - static_cast<uint32_t>(v_warp + w));
             }
           }
         }
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&sh.acc_empty[a]);
+      if (lane == 0) mbar_arrive_remote(acc_empty0 + static_cast<uint32_t>(a * sizeof(unsigned long long)));
     }
-    if (!kWriteLogits && valid && !sh.abort) {
-      const unsigned long long key = best_i < 0 ? 0ull : make_key(best, static_cast<uint32_t>(best_i));
-      if (key) atomicMax(&p.row_key[tok], key);
-      if (has_zx) p.draft_logit[tok] = zx;
-      if (nan_acc != nan_acc) atomicOr(&p.flags[tok / K1], ASD_STATUS_NAN_LOGIT);
+    if (!kWriteLogits && !sh.abort) {
+#pragma unroll
+      for (int c = 0; c < kChunks; ++c) {
+        const int tok = m * kTN + c * 32 + lane;
+        const unsigned long long key = best[c];
+        if (tok < q.T && key) {
+          atomicMax(&p.row_key[tok], key);
+          if ((key >> 32) == 0xffc00000ull) atomicOr(&p.flags[tok / K1], ASD_STATUS_NAN_LOGIT);
+        }
+      }
     }
     __threadfence();
   }
 
   tc_fence_before();
   __syncthreads();
-  if (sh.abort && warp == 0 && lane == 0) {
-    // wait (bounded) for the loads still in flight before the CTA exits
+  if (sh.abort && leader && warp == 0 && lane == 0) {
+    // wait (bounded) for the loads still in flight before the pair exits
     for (int it = it_issued > kStages ? it_issued - kStages : 0; it < it_issued; ++it) {
       const int s = it % kStages;
       const unsigned long long t0 = global_ns();
-      while (!mbar_try_wait(&sh.full[s], (it / kStages) & 1) && global_ns() - t0 < kWaitLimitNs) {
+      while (!mbar_try_wait_cluster(&sh.full[s], (it / kStages) & 1) && global_ns() - t0 < kWaitLimitNs) {
       }
     }
   }
   __syncthreads();
+  cluster_sync_all();  // neither CTA frees tensor memory or exits while the other may still use the pair
   if (warp == 1) {
     tc_fence_after();
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
   }
   if (kWriteLogits || sh.abort) return;
 
   // Count this CTA's rows of each request of its token tile; the CTA that
   // completes a request (every CTA of the tile has counted) runs its selection.
-  const int K1 = p.K + 1;
-  const int t0 = m * kBM, t1 = (m + 1) * kBM < q.T ? (m + 1) * kBM : q.T;
+  const int t0 = m * kTN, t1 = (m + 1) * kTN < q.T ? (m + 1) * kTN : q.T;
   if (t0 < t1) {
     const int b_first = t0 / K1, b_last = (t1 - 1) / K1;
-    const unsigned long long total = static_cast<unsigned long long>(K1) * q.ctas_per_tile;
+    const unsigned long long total = static_cast<unsigned long long>(K1) * 2ull * q.pairs_per_tile;
     for (int b = b_first + warp; b <= b_last; b += kLmThreads / 32) {
       const int r0 = b * K1 > t0 ? b * K1 : t0;
       const int r1 = (b + 1) * K1 < t1 ? (b + 1) * K1 : t1;
@@ -364,7 +517,7 @@ EncodeTiledFn encode_tiled() {
   return fn;
 }
 
-// 2-D bf16 row-major [rows, cols] tensor, boxes of box_rows x 64 columns,
+// 2-D bf16 row-major [rows, cols] tensor, boxes of box_rows x kBK columns,
 // 128-byte swizzle; out-of-range rows and columns read as zero.
 bool make_map(CUtensorMap* map, const void* ptr, int rows, int cols, int box_rows) {
   EncodeTiledFn fn = encode_tiled();
@@ -381,7 +534,7 @@ bool make_map(CUtensorMap* map, const void* ptr, int rows, int cols, int box_row
 struct LmDevice {
   int sms = 0;
   int major = 0, minor = 0;
-  bool ready[4] = {false, false, false, false};
+  int pairs[4] = {0, 0, 0, 0};  // CTA pairs resident at once, per kernel instance (0: not set up yet)
 };
 
 int lm_device(LmDevice** out) {
@@ -402,6 +555,21 @@ int lm_device(LmDevice** out) {
   return ASD_OK;
 }
 
+cudaLaunchConfig_t pair_config(unsigned grid, cudaStream_t stream, cudaLaunchAttribute* attr) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid, 1, 1);
+  cfg.blockDim = dim3(kLmThreads, 1, 1);
+  cfg.dynamicSmemBytes = kLmSmemBytes;
+  cfg.stream = stream;
+  attr->id = cudaLaunchAttributeClusterDimension;
+  attr->val.clusterDim.x = 2;
+  attr->val.clusterDim.y = 1;
+  attr->val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cfg;
+}
+
 template <bool kStrict, bool kWriteLogits>
 int launch_lmhead(const void* hidden, const void* weight, int H, int T, VerifyParams& p, float* logits_out,
                   cudaStream_t stream) {
@@ -411,27 +579,32 @@ int launch_lmhead(const void* hidden, const void* weight, int H, int T, VerifyPa
   if (dev->major != 10) return ASD_ERR_DEVICE;  // tcgen05 needs a Blackwell (sm_10x) device
   auto kernel = lmhead_verify_kernel<kStrict, kWriteLogits>;
   const int slot = (kStrict ? 1 : 0) + (kWriteLogits ? 2 : 0);
-  if (!dev->ready[slot]) {
+  cudaLaunchAttribute attr;
+  if (dev->pairs[slot] == 0) {
     if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kLmSmemBytes)) !=
         cudaSuccess)
       return ASD_ERR_CUDA;
-    dev->ready[slot] = true;
+    cudaLaunchConfig_t probe = pair_config(static_cast<unsigned>(dev->sms & ~1), stream, &attr);
+    int clusters = 0;
+    if (cudaOccupancyMaxActiveClusters(&clusters, kernel, &probe) != cudaSuccess || clusters < 1)
+      return ASD_ERR_CUDA;
+    dev->pairs[slot] = clusters;
   }
   CUtensorMap map_h, map_w;
-  if (!make_map(&map_h, hidden, T, H, kBM) || !make_map(&map_w, weight, p.V, H, kBN)) return ASD_ERR_CUDA;
+  if (!make_map(&map_h, hidden, T, H, kHalfN) || !make_map(&map_w, weight, p.V, H, kHalfM)) return ASD_ERR_CUDA;
   LmParams q;
   q.T = T;
   q.H = H;
   q.V = p.V;
-  q.token_tiles = (T + kBM - 1) / kBM;
-  q.ctas_per_tile = dev->sms / q.token_tiles > 0 ? dev->sms / q.token_tiles : 1;
-  q.vocab_tiles = (p.V + kBN - 1) / kBN;
-  if (q.ctas_per_tile > q.vocab_tiles) q.ctas_per_tile = q.vocab_tiles;
+  q.token_tiles = (T + kTN - 1) / kTN;
+  q.pairs_per_tile = dev->pairs[slot] / q.token_tiles > 0 ? dev->pairs[slot] / q.token_tiles : 1;
+  q.vocab_tiles = (p.V + kPairM - 1) / kPairM;
+  if (q.pairs_per_tile > q.vocab_tiles) q.pairs_per_tile = q.vocab_tiles;
   q.k_steps = (H + kBK - 1) / kBK;
   q.logits_out = logits_out;
-  const unsigned grid = static_cast<unsigned>(q.token_tiles * q.ctas_per_tile);
-  kernel<<<grid, kLmThreads, kLmSmemBytes, stream>>>(map_h, map_w, p, q);
-  return cudaGetLastError() == cudaSuccess ? ASD_OK : ASD_ERR_CUDA;
+  const unsigned grid = 2u * static_cast<unsigned>(q.token_tiles * q.pairs_per_tile);
+  cudaLaunchConfig_t cfg = pair_config(grid, stream, &attr);
+  return cudaLaunchKernelEx(&cfg, kernel, map_h, map_w, p, q) == cudaSuccess ? ASD_OK : ASD_ERR_CUDA;
 }
 
 int check_lm_inputs(const void* hidden, const void* weight, int H) {
