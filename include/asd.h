@@ -102,6 +102,17 @@ int asd_workspace_init(void* workspace, size_t bytes, asd_stream_t stream);
  * incomplete and the workspace must be re-initialised with asd_workspace_init. */
 int asd_workspace_error(const void* workspace, int* error, asd_stream_t stream);
 
+/* Self-test of the failure detection above (the paper has no counterpart):
+ * launches one CTA whose thread waits, with the same bounded mbarrier wait as
+ * the pipeline kernels, on a barrier that nothing signals. After about one
+ * second the wait gives up, the kernel writes ASD_ERR_TIMEOUT to the
+ * workspace's error word and returns; nothing faults and the context stays
+ * usable. `workspace` is any workspace of at least 4 bytes (16-byte aligned);
+ * read the result with asd_workspace_error and re-initialise the workspace
+ * before its next verify call. Returns ASD_ERR_NULL / ASD_ERR_WORKSPACE /
+ * ASD_ERR_ALIGN on bad arguments, ASD_ERR_CUDA if the launch fails. */
+int asd_selftest_wait_timeout(void* workspace, size_t workspace_bytes, asd_stream_t stream);
+
 /*
  * ASD verification of B draft blocks (Eq. 1, 3, 5-13; Alg. 1).
  *

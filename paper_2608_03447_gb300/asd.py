@@ -52,6 +52,8 @@ def _declare(lib: ctypes.CDLL) -> ctypes.CDLL:
     lib.asd_workspace_init.restype = i32
     lib.asd_workspace_error.argtypes = [vp, ctypes.POINTER(i32), vp]
     lib.asd_workspace_error.restype = i32
+    lib.asd_selftest_wait_timeout.argtypes = [vp, sz, vp]
+    lib.asd_selftest_wait_timeout.restype = i32
     lib.asd_verify.argtypes = [vp, i32, i32, i32, i32, vp, vp, f32, i32, vp, vp, vp, vp, vp, vp, vp, sz, vp]
     lib.asd_verify.restype = i32
     lib.asd_verify_strict.argtypes = [vp, i32, i32, i32, i32, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
@@ -176,6 +178,17 @@ class Workspace:
         word = ctypes.c_int(0)
         _check("asd_workspace_error", load().asd_workspace_error(self.ptr, ctypes.byref(word), _stream(stream)))
         return word.value
+
+    def reset(self, stream=None) -> None:
+        """Zero the workspace again (asd_workspace_init), e.g. after a non-zero error word."""
+        _check("asd_workspace_init", load().asd_workspace_init(self.ptr, self.nbytes, _stream(stream)))
+
+
+def selftest_wait_timeout(workspace: "Workspace", stream=None) -> None:
+    """asd_selftest_wait_timeout: a bounded wait on a barrier nothing signals (about one second); the
+    workspace's error word then reads ASD_ERR_TIMEOUT."""
+    _check("asd_selftest_wait_timeout", load().asd_selftest_wait_timeout(workspace.ptr, workspace.nbytes,
+                                                                         _stream(stream)))
 
 
 def make_ledger(B: int, budget: float, spent: float = 0.0, device="cuda") -> torch.Tensor:

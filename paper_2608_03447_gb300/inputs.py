@@ -25,6 +25,17 @@ against a background logit spread of 0.02 * sqrt(H) = 1.43) and
 beta' = beta - U(0, 0.7) in 20 % of rows, beta - U(1, 4) otherwise; cast to
 bf16. Drafts use the same p_hit / p_near / uniform mix over (p, p', uniform).
 
+Exactly representable fused LM-head inputs (parity without tolerances): W and
+h hold integers in {-1, 0, 1}, so every product and every partial sum is an
+integer far below 2^24 and the fp32 logits are exact whatever the summation
+order. Sixteen source rows of W are copied to rows at distances 1, 40, 130
+and 600 (the same warp, another warp, the other SM of a pair, another pair of
+the 2-SM kernel's tiling), so exact ties cross every level of the reduction.
+Token t copies W[p_t] on a random 75 % of its coordinates (zeros elsewhere),
+p_t a source row with probability 1/2, else uniform; drafts are p_t with
+probability 0.6, else uniform. Where p_t has a lower-indexed copy the draft
+differs from the target's token with zero regret.
+
 Seeds: seed = 1000 * config + 17 * point + block.
 """
 from __future__ import annotations
@@ -141,6 +152,32 @@ def gen_lmhead(B: int, K: int, H: int, V: int, seed: int, device="cpu",
     p = planted[pos_rows]
     draft = torch.where(u < p_hit, p[:, :, 0], torch.where(u < p_hit + p_near, p[:, :, 1], uniform))
     return LMHeadInputs(hidden=hidden, weight=W, draft=draft.to(torch.int32).contiguous())
+
+
+TIE_OFFSETS = (1, 40, 130, 600)
+
+
+def gen_lmhead_exact(B: int, K: int, H: int, V: int, seed: int, device="cpu") -> LMHeadInputs:
+    """Integer-valued fused LM-head inputs with planted exact ties (see the module docstring)."""
+    dev = torch.device(device)
+    g = _generator(torch.device("cpu"), seed)
+    T = B * (K + 1)
+    W = torch.randint(-1, 2, (V, H), generator=g).float()
+    sources = torch.randint(0, V, (16,), generator=g)
+    for src in sources.tolist():
+        for off in TIE_OFFSETS:
+            if src + off < V:
+                W[src + off] = W[src]
+    pick_src = torch.rand(T, generator=g) < 0.5
+    p = torch.where(pick_src, sources[torch.randint(0, 16, (T,), generator=g)], torch.randint(0, V, (T,), generator=g))
+    keep = torch.rand(T, H, generator=g) < 0.75
+    h = torch.where(keep, W[p], torch.zeros(()))
+    pos_rows = (torch.arange(B)[:, None] * (K + 1) + torch.arange(K)[None, :])
+    u = torch.rand(B, K, generator=g)
+    draft = torch.where(u < 0.6, p[pos_rows], torch.randint(0, V, (B, K), generator=g))
+    return LMHeadInputs(hidden=h.to(torch.bfloat16).contiguous().to(dev),
+                        weight=W.to(torch.bfloat16).contiguous().to(dev),
+                        draft=draft.to(torch.int32).contiguous().to(dev))
 
 
 # The five workloads (sizes from the paper's settings: Qwen3 vocabulary 151936,

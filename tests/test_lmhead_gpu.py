@@ -157,3 +157,56 @@ def test_lmhead_full_size_sampled(asd):
     z64, z32 = oracle_logits(inp.hidden, inp.weight, tokens)
     n_ok, n = compare(out, z64, z32, inp.draft, tokens, B, K, cfg["gate"], cfg["cap"], cfg["budget"])
     assert n_ok >= 1
+
+
+@pytest.mark.parametrize("B,K,H,V", [(8, 8, 512, 1000), (40, 8, 256, 2100), (5, 0, 64, 777), (3, 16, 320, 1300)])
+def test_lmhead_verify_exact_inputs_bit_exact(asd, B, K, H, V):
+    """Integer h and W: the fp32 logits are exact, so every output equals the oracle's bit for bit,
+    ties across warps, SMs and SM pairs included (lowest index wins)."""
+    inp = inputs.gen_lmhead_exact(B, K, H, V, 7000 + B + K + H, "cuda")
+    ledger0 = torch.tensor([[8.0, 0.0]] * B, dtype=torch.float32)
+    led = ledger0.cuda()
+    out = asd.lmhead_verify(inp.hidden, inp.weight, inp.draft, led, 1.0, 2)
+    torch.cuda.synchronize()
+    T = B * (K + 1)
+    z64, z32 = oracle_logits(inp.hidden, inp.weight, range(T))
+    assert np.array_equal(z64, z32.astype(np.float64)), "integer inputs must give exact logits"
+    o = oracle.verify(z32.reshape(B, K + 1, V), inp.draft.cpu().numpy(), ledger0.numpy(), 1.0, 2)
+    assert np.array_equal(out["row_argmax"].cpu().numpy(), o["row_argmax"])
+    assert np.array_equal(out["row_top"].cpu().numpy(), z32.reshape(B, K + 1, V).max(axis=2))
+    assert np.array_equal(out["row_regret"].cpu().numpy().view(np.int32), o["row_regret"].view(np.int32))
+    assert np.array_equal(out["accepted_len"].cpu().numpy(), o["accepted_len"])
+    assert np.array_equal(out["committed"].cpu().numpy(), o["committed"])
+    assert np.array_equal(out["recovery"].cpu().numpy(), o["recovery"])
+    assert np.array_equal(led.cpu().numpy().view(np.int32), o["ledger"].view(np.int32))
+    assert np.array_equal(out["status"].cpu().numpy(), o["status"])
+    # the planted copies do produce ties that the lowest index has to win
+    zr = z32.reshape(T, V)
+    ties = int(((zr == zr.max(axis=1, keepdims=True)).sum(axis=1) > 1).sum())
+    assert ties > 0
+
+
+def test_lmhead_verify_nan_row_flags_its_request(asd):
+    """A NaN hidden state makes every logit of its row NaN: that request is flagged and left alone
+    (a = 0, ledger unchanged); every other request matches the oracle exactly."""
+    B, K, H, V = 6, 4, 128, 900
+    inp = inputs.gen_lmhead_exact(B, K, H, V, 7100, "cuda")
+    bad_row = 2 * (K + 1) + 3  # request 2, row 3
+    hidden = inp.hidden.clone()
+    hidden[bad_row, 5] = float("nan")
+    ledger0 = torch.tensor([[8.0, 0.5]] * B, dtype=torch.float32)
+    led = ledger0.cuda()
+    out = asd.lmhead_verify(hidden, inp.weight, inp.draft, led, 1.0, 2)
+    torch.cuda.synchronize()
+    z64, z32 = oracle_logits(hidden, inp.weight, range(B * (K + 1)))
+    assert np.isnan(z32[bad_row]).all()
+    o = oracle.verify(z32.reshape(B, K + 1, V), inp.draft.cpu().numpy(), ledger0.numpy(), 1.0, 2)
+    st = out["status"].cpu().numpy()
+    assert st[2] & oracle.STATUS_NAN_LOGIT and o["status"][2] & oracle.STATUS_NAN_LOGIT
+    assert out["accepted_len"][2].item() == 0
+    assert np.array_equal(led.cpu().numpy()[2], ledger0.numpy()[2])
+    for b in [0, 1, 3, 4, 5]:
+        assert st[b] == o["status"][b] == 0
+        assert out["accepted_len"][b].item() == o["accepted_len"][b]
+        assert np.array_equal(out["committed"][b].cpu().numpy(), o["committed"][b])
+        assert np.array_equal(led.cpu().numpy()[b].view(np.int32), o["ledger"][b].view(np.int32))

@@ -307,3 +307,33 @@ def test_verify_reads_pinned_host_memory_in_place(asd, kernel):
         asd.host_alias(torch.zeros(4))  # the binding insists on pinned tensors
     alias = ctypes.c_void_p(0)
     assert asd.load().asd_host_alias(hl.data_ptr(), ctypes.byref(alias)) == 0 and alias.value
+
+
+ERR_TIMEOUT = 9  # ASD_ERR_TIMEOUT
+
+
+def test_bounded_wait_reports_timeout_and_context_survives(asd):
+    """Failure detection without a fault: a bounded wait on a barrier that nothing signals gives up
+    after about a second, the workspace's error word reads ASD_ERR_TIMEOUT, and the same context and
+    workspace then verify a block correctly once the workspace is re-initialised."""
+    import time
+    B, K, V = 4, 8, 1024
+    ws = asd.Workspace(B, K, V, 0)
+    assert ws.error() == 0
+    t0 = time.perf_counter()
+    asd.selftest_wait_timeout(ws)
+    assert ws.error() == ERR_TIMEOUT
+    elapsed = time.perf_counter() - t0
+    assert 0.5 < elapsed < 30.0, f"the wait should give up after about a second, took {elapsed:.2f} s"
+    ws.reset()
+    assert ws.error() == 0
+    block = inputs.gen_block(B, K, V, torch.float32, 4321, "cuda")
+    led = asd.make_ledger(B, 4.0)
+    led0 = led.cpu().numpy()
+    out = asd.verify(block.logits, block.draft, led, 1.0, 2, workspace=ws)
+    torch.cuda.synchronize()
+    o = oracle.verify(block.logits.cpu().numpy(), block.draft.cpu().numpy(), led0, 1.0, 2)
+    assert ws.error() == 0
+    assert np.array_equal(out["accepted_len"].cpu().numpy(), o["accepted_len"])
+    assert np.array_equal(out["committed"].cpu().numpy(), o["committed"])
+    assert np.array_equal(led.cpu().numpy().view(np.int32), o["ledger"].view(np.int32))
