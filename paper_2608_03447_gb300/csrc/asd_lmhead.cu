@@ -29,6 +29,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
 #include <cstdlib>
 #include <mutex>
 
@@ -534,7 +535,9 @@ bool make_map(CUtensorMap* map, const void* ptr, int rows, int cols, int box_row
 struct LmDevice {
   int sms = 0;
   int major = 0, minor = 0;
-  int pairs[4] = {0, 0, 0, 0};  // CTA pairs resident at once, per kernel instance (0: not set up yet)
+  // CTA pairs resident at once, per kernel instance (0: not set up yet); the
+  // set-up is idempotent, so two threads racing to do it store the same value
+  std::atomic<int> pairs[4] = {};
 };
 
 int lm_device(LmDevice** out) {
@@ -580,15 +583,14 @@ int launch_lmhead(const void* hidden, const void* weight, int H, int T, VerifyPa
   auto kernel = lmhead_verify_kernel<kStrict, kWriteLogits>;
   const int slot = (kStrict ? 1 : 0) + (kWriteLogits ? 2 : 0);
   cudaLaunchAttribute attr;
-  if (dev->pairs[slot] == 0) {
+  int pairs = dev->pairs[slot].load(std::memory_order_acquire);
+  if (pairs == 0) {
     if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kLmSmemBytes)) !=
         cudaSuccess)
       return ASD_ERR_CUDA;
     cudaLaunchConfig_t probe = pair_config(static_cast<unsigned>(dev->sms & ~1), stream, &attr);
-    int clusters = 0;
-    if (cudaOccupancyMaxActiveClusters(&clusters, kernel, &probe) != cudaSuccess || clusters < 1)
-      return ASD_ERR_CUDA;
-    dev->pairs[slot] = clusters;
+    if (cudaOccupancyMaxActiveClusters(&pairs, kernel, &probe) != cudaSuccess || pairs < 1) return ASD_ERR_CUDA;
+    dev->pairs[slot].store(pairs, std::memory_order_release);
   }
   CUtensorMap map_h, map_w;
   if (!make_map(&map_h, hidden, T, H, kHalfN) || !make_map(&map_w, weight, p.V, H, kHalfM)) return ASD_ERR_CUDA;
@@ -597,7 +599,7 @@ int launch_lmhead(const void* hidden, const void* weight, int H, int T, VerifyPa
   q.H = H;
   q.V = p.V;
   q.token_tiles = (T + kTN - 1) / kTN;
-  q.pairs_per_tile = dev->pairs[slot] / q.token_tiles > 0 ? dev->pairs[slot] / q.token_tiles : 1;
+  q.pairs_per_tile = pairs / q.token_tiles > 0 ? pairs / q.token_tiles : 1;
   q.vocab_tiles = (p.V + kPairM - 1) / kPairM;
   if (q.pairs_per_tile > q.vocab_tiles) q.pairs_per_tile = q.vocab_tiles;
   q.k_steps = (H + kBK - 1) / kBK;

@@ -24,6 +24,7 @@
 #include <stdint.h>
 
 #include <cstdlib>
+#include <atomic>
 #include <mutex>
 
 #include "asd.h"
@@ -772,7 +773,9 @@ int resident_warps(int* out) {
 
 struct DeviceInfo {
   int sms = 0;
-  bool tma_ready[8] = {false, false, false, false, false, false, false, false};
+  // set once the TMA kernel instance has its shared-memory opt-in; the
+  // opt-in is idempotent, so two threads racing to set it up is harmless
+  std::atomic<bool> tma_ready[8] = {};
 };
 
 // The TMA path's selection runs in its own kernel right behind the row stage
@@ -818,12 +821,12 @@ int launch_tma(VerifyParams& p, cudaStream_t stream) {
   if (rc != ASD_OK) return rc;
   const bool split = use_split();
   const int slot = (sizeof(T) == 2 ? 2 : 0) + (kStrict ? 1 : 0) + (split ? 4 : 0);
-  if (!info->tma_ready[slot]) {
+  if (!info->tma_ready[slot].load(std::memory_order_acquire)) {
     auto kernel = split ? verify_tma_kernel<T, kStrict, true> : verify_tma_kernel<T, kStrict, false>;
     if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(sizeof(TmaShared))) != cudaSuccess)
       return ASD_ERR_CUDA;
-    info->tma_ready[slot] = true;
+    info->tma_ready[slot].store(true, std::memory_order_release);
   }
   long long ncta = (bulk + kMinPerCta - 1) / kMinPerCta;
   if (ncta > info->sms) ncta = info->sms;
