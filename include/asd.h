@@ -60,6 +60,18 @@ typedef struct {
 /* Logit storage types. */
 enum { ASD_F32 = 0, ASD_BF16 = 1 };
 
+/* Flag ORed into the dtype argument of the verify entry points: the logits and
+ * draft tokens are resident, i.e. no kernel that is still running or queued
+ * ahead of this call on the stream writes them (they were written by work that
+ * has completed, by a copy, or by the host). The row stage then starts
+ * streaming them while the previous kernel on the stream finishes (programmatic
+ * dependent launch), which overlaps consecutive calls. Without the flag the row
+ * stage still launches early but reads nothing before the previous kernel has
+ * completed and its writes are visible, so a producer kernel (such as the
+ * model's LM head) may write the logits right before the call. Results are the
+ * same either way; only the overlap differs. */
+#define ASD_RESIDENT_INPUTS 0x100
+
 /* Return codes. */
 enum {
   ASD_OK = 0,
@@ -133,6 +145,7 @@ int asd_selftest_wait_timeout(void* workspace, size_t workspace_bytes, asd_strea
  * status        [B]       ASD_STATUS_* bits; may be NULL
  * workspace     >= asd_workspace_size(...) bytes, 16-byte aligned, zeroed
  *               by asd_workspace_init before first use
+ * dtype         ASD_F32 or ASD_BF16, optionally | ASD_RESIDENT_INPUTS (above)
  *
  * Arithmetic (all fp32, round to nearest): argmax by IEEE comparison
  * (-0 == +0), then per request, left to right over the mismatches d_j = 1:
@@ -173,7 +186,11 @@ int asd_verify_strict(const void* logits, int dtype, int B, int K, int V, const 
  * devices get ASD_ERR_DEVICE.
  * Precision: the logits are fp32 sums of bf16 products in the tensor core's
  * order, so ties and near-ties (within about 1e-5 of the row's scale) may
- * resolve differently from an exact (fp64) evaluation.
+ * resolve differently from an exact (fp64) evaluation; exact ties between
+ * equal fp32 logits go to the lowest index, as in asd_verify.
+ * Launch: clusters of two CTAs, one per SM of a pair, each with about 200 KB
+ * of shared memory and all 512 tensor-memory columns of its SM, so a call
+ * occupies the GPU's SM pairs while it runs.
  */
 int asd_lmhead_workspace_size(int B, int K, int V, int H, size_t* bytes);
 int asd_lmhead_verify(const void* hidden, const void* weight, int H, int B, int K, int V,

@@ -32,6 +32,7 @@ STATUS_NAN_LOGIT = 2
 STATUS_BAD_LEDGER = 4
 STATUS_OVERFLOW = 8
 MAX_K = 31
+RESIDENT_INPUTS = 0x100  # ASD_RESIDENT_INPUTS, ORed into the dtype code
 INT32_MAX = 2**31 - 1
 
 _lock = threading.Lock()
@@ -131,6 +132,10 @@ def _stream(stream) -> int:
     return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
 
 
+def _flag(resident: bool) -> int:
+    return RESIDENT_INPUTS if resident else 0
+
+
 def _dtype_code(t: torch.Tensor) -> int:
     if t.dtype == torch.float32:
         return F32
@@ -222,15 +227,20 @@ def _shape(logits: torch.Tensor, draft: torch.Tensor):
 
 
 def verify(logits: torch.Tensor, draft: torch.Tensor, ledger: torch.Tensor, gate: float, cap: int,
-           workspace: Workspace | None = None, out: dict | None = None, stream=None) -> dict:
-    """asd_verify: ASD verification of a batch of draft blocks; updates ``ledger`` in place."""
+           workspace: Workspace | None = None, out: dict | None = None, stream=None, resident: bool = False) -> dict:
+    """asd_verify: ASD verification of a batch of draft blocks; updates ``ledger`` in place.
+
+    ``resident=True`` passes ASD_RESIDENT_INPUTS: no kernel still running or queued ahead on the stream
+    writes ``logits`` or ``draft``, so the row stage may stream them while the previous kernel finishes.
+    """
     B, K, V = _shape(logits, draft)
     if ledger.shape != (B, 2) or ledger.dtype != torch.float32 or not ledger.is_contiguous():
         raise ValueError("ledger must be a contiguous float32 tensor [B, 2] of (budget, spent)")
     code = _dtype_code(logits)
     ws = workspace or Workspace(B, K, V, code, logits.device, stream)
     o = out or alloc_outputs(B, K, logits.device)
-    rc = load().asd_verify(_ptr(logits), code, B, K, V, _ptr(draft), _ptr(ledger), float(gate), int(cap),
+    rc = load().asd_verify(_ptr(logits), code | _flag(resident), B, K, V, _ptr(draft), _ptr(ledger), float(gate),
+                           int(cap),
                            _ptr(o["accepted_len"]), _ptr(o["committed"]), _ptr(o["recovery"]),
                            _ptr(o.get("row_argmax")), _ptr(o.get("row_regret")), _ptr(o.get("status")),
                            ws.ptr, ws.nbytes, _stream(stream))
@@ -239,7 +249,7 @@ def verify(logits: torch.Tensor, draft: torch.Tensor, ledger: torch.Tensor, gate
 
 
 def verify_noalloc(logits: torch.Tensor, draft: torch.Tensor, ledger: torch.Tensor, gate: float, cap: int,
-                   out: dict | None = None, stream=None) -> dict:
+                   out: dict | None = None, stream=None, resident: bool = False) -> dict:
     """asd_verify_noalloc: asd_verify with the library's fixed scratch instead of a workspace.
 
     For callers that may not allocate device memory while verifying. Calls that
@@ -249,7 +259,8 @@ def verify_noalloc(logits: torch.Tensor, draft: torch.Tensor, ledger: torch.Tens
     if ledger.shape != (B, 2) or ledger.dtype != torch.float32 or not ledger.is_contiguous():
         raise ValueError("ledger must be a contiguous float32 tensor [B, 2] of (budget, spent)")
     o = out or alloc_outputs(B, K, logits.device)
-    rc = load().asd_verify_noalloc(_ptr(logits), _dtype_code(logits), B, K, V, _ptr(draft), _ptr(ledger),
+    rc = load().asd_verify_noalloc(_ptr(logits), _dtype_code(logits) | _flag(resident), B, K, V, _ptr(draft),
+                                   _ptr(ledger),
                                    float(gate), int(cap), _ptr(o["accepted_len"]), _ptr(o["committed"]),
                                    _ptr(o["recovery"]), _ptr(o.get("row_argmax")), _ptr(o.get("row_regret")),
                                    _ptr(o.get("status")), _stream(stream))
@@ -258,13 +269,13 @@ def verify_noalloc(logits: torch.Tensor, draft: torch.Tensor, ledger: torch.Tens
 
 
 def verify_strict(logits: torch.Tensor, draft: torch.Tensor, workspace: Workspace | None = None,
-                  out: dict | None = None, stream=None) -> dict:
+                  out: dict | None = None, stream=None, resident: bool = False) -> dict:
     """asd_verify_strict: strict greedy verification (Eq. 2)."""
     B, K, V = _shape(logits, draft)
     code = _dtype_code(logits)
     ws = workspace or Workspace(B, K, V, code, logits.device, stream)
     o = out or alloc_outputs(B, K, logits.device)
-    rc = load().asd_verify_strict(_ptr(logits), code, B, K, V, _ptr(draft),
+    rc = load().asd_verify_strict(_ptr(logits), code | _flag(resident), B, K, V, _ptr(draft),
                                   _ptr(o["accepted_len"]), _ptr(o["committed"]), _ptr(o["recovery"]),
                                   _ptr(o.get("row_argmax")), _ptr(o.get("row_regret")), _ptr(o.get("status")),
                                   ws.ptr, ws.nbytes, _stream(stream))
@@ -283,7 +294,8 @@ def _alias(t: torch.Tensor) -> int:
 
 
 def verify_from_host(logits_host: torch.Tensor, draft_host: torch.Tensor, ledger: torch.Tensor, gate: float,
-                     cap: int, workspace: Workspace, out: dict, host_out: dict, stream=None) -> dict:
+                     cap: int, workspace: Workspace, out: dict, host_out: dict, stream=None,
+                     resident: bool = False) -> dict:
     """End-to-end step from pinned host buffers: verify reading them in place, copy the results out.
 
     The kernels read the pinned logits and drafts through their device aliases
@@ -297,7 +309,8 @@ def verify_from_host(logits_host: torch.Tensor, draft_host: torch.Tensor, ledger
     B, K1, V = logits_host.shape
     K = K1 - 1
     code = _dtype_code(logits_host)
-    rc = load().asd_verify(_alias(logits_host), code, B, K, V, _alias(draft_host), _ptr(ledger), float(gate),
+    rc = load().asd_verify(_alias(logits_host), code | _flag(resident), B, K, V, _alias(draft_host), _ptr(ledger),
+                           float(gate),
                            int(cap), _ptr(out["accepted_len"]), _ptr(out["committed"]), _ptr(out["recovery"]),
                            _ptr(out.get("row_argmax")), _ptr(out.get("row_regret")), _ptr(out.get("status")),
                            workspace.ptr, workspace.nbytes, _stream(stream))
@@ -367,7 +380,8 @@ def blocks_workspace(nblk: int, B: int, K: int, V: int, dtype: int, device=None,
 
 
 def verify_blocks(logits: torch.Tensor, draft: torch.Tensor, ledger: torch.Tensor, gate: float, cap: int,
-                  workspace: Workspace | None = None, out: dict | None = None, stream=None) -> dict:
+                  workspace: Workspace | None = None, out: dict | None = None, stream=None,
+                  resident: bool = False) -> dict:
     """asd_verify_blocks: nblk sequential blocks of the same requests in one call.
 
     logits [nblk, B, K+1, V], draft [nblk, B, K], ledger [B, 2]; outputs carry a
@@ -386,7 +400,8 @@ def verify_blocks(logits: torch.Tensor, draft: torch.Tensor, ledger: torch.Tenso
     if out is None:
         flat = alloc_outputs(nblk * B, K, logits.device)
         out = {k: v.view(nblk, B, *v.shape[1:]) for k, v in flat.items()}
-    rc = load().asd_verify_blocks(_ptr(logits), code, nblk, B, K, V, _ptr(draft), _ptr(ledger), float(gate),
+    rc = load().asd_verify_blocks(_ptr(logits), code | _flag(resident), nblk, B, K, V, _ptr(draft), _ptr(ledger),
+                                  float(gate),
                                   int(cap), _ptr(out["accepted_len"]), _ptr(out["committed"]), _ptr(out["recovery"]),
                                   _ptr(out.get("row_argmax")), _ptr(out.get("row_regret")), _ptr(out.get("status")),
                                   ws.ptr, ws.nbytes, _stream(stream))
@@ -416,7 +431,8 @@ PARTIAL_WORDS = 6  # asd_partial: uint64 key, float top, float draft_logit, uint
 
 
 def shard_partials(logits: torch.Tensor, draft: torch.Tensor, v_offset: int, V: int,
-                   workspace: Workspace | None = None, out: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+                   workspace: Workspace | None = None, out: torch.Tensor | None = None, stream=None,
+                   resident: bool = False) -> torch.Tensor:
     """asd_shard_partials: one vocabulary shard's per-row partials, as int32 [B*(K+1), 6] (asd_partial).
 
     logits [B, K+1, Vs] hold vocabulary entries v_offset .. v_offset+Vs-1 of V; draft holds global ids.
@@ -425,7 +441,8 @@ def shard_partials(logits: torch.Tensor, draft: torch.Tensor, v_offset: int, V: 
     code = _dtype_code(logits)
     ws = workspace or Workspace(B, K, Vs, code, logits.device, stream)
     o = out if out is not None else torch.empty(B * (K + 1), PARTIAL_WORDS, dtype=torch.int32, device=logits.device)
-    rc = load().asd_shard_partials(_ptr(logits), code, B, K, Vs, int(v_offset), int(V), _ptr(draft), _ptr(o),
+    rc = load().asd_shard_partials(_ptr(logits), code | _flag(resident), B, K, Vs, int(v_offset), int(V), _ptr(draft),
+                                   _ptr(o),
                                    ws.ptr, ws.nbytes, _stream(stream))
     _check("asd_shard_partials", rc)
     return o

@@ -40,6 +40,8 @@ struct VerifyParams {
   int v_offset;                 // vocabulary shard: global index of this shard's entry 0 (else 0)
   int v_total;                  // vocabulary shard: entries of the whole vocabulary (else V)
   asd_partial* partials;        // vocabulary shard: [B*(K+1)] outputs instead of the selection
+  int resident;                 // ASD_RESIDENT_INPUTS: logits and drafts may be read before the
+                                // previous launch on the stream has completed
 };
 
 // ---------------------------------------------------------------- element access
@@ -393,7 +395,11 @@ inline WorkspaceLayout layout_for(int B, int K) {
   return l;
 }
 
+// The storage type of a dtype argument (without ASD_RESIDENT_INPUTS).
+inline int dtype_code(int dtype) { return dtype & ~ASD_RESIDENT_INPUTS; }
+
 inline int check_shape(int B, int K, int V, int dtype) {
+  dtype = dtype_code(dtype);
   if (dtype != ASD_F32 && dtype != ASD_BF16) return ASD_ERR_DTYPE;
   if (B < 0 || K < 0 || K > ASD_MAX_K || V < 1) return ASD_ERR_SHAPE;
   return ASD_OK;

@@ -25,6 +25,7 @@
 
 #include <cstdlib>
 #include <atomic>
+#include <cstring>
 #include <mutex>
 
 #include "asd.h"
@@ -79,7 +80,7 @@ __device__ __forceinline__ float vec_max(const uint4& v, __nv_bfloat16) {
 
 // Reduces elements [s0, s1) of one row (which starts at flat index row0) to a
 // key; every lane returns the warp's key. Sets *nan when a NaN was seen.
-template <typename T>
+template <typename T, int kU = kUnroll>
 __device__ __forceinline__ unsigned long long segment_key(const T* z, long long s0, long long s1,
                                                           long long row0, long long head,
                                                           int lane, bool* nan) {
@@ -104,12 +105,12 @@ __device__ __forceinline__ unsigned long long segment_key(const T* z, long long 
     int bvec = -1;
     uint4 saved = make_uint4(0, 0, 0, 0);
     long long k = lane;
-    for (; k + 32 * (kUnroll - 1) < nvec; k += 32 * kUnroll) {
-      uint4 v[kUnroll];
+    for (; k + 32 * (kU - 1) < nvec; k += 32 * kU) {
+      uint4 v[kU];
 #pragma unroll
-      for (int u = 0; u < kUnroll; ++u) v[u] = load_stream(vp + k + 32 * u);
+      for (int u = 0; u < kU; ++u) v[u] = load_stream(vp + k + 32 * u);
 #pragma unroll
-      for (int u = 0; u < kUnroll; ++u) {
+      for (int u = 0; u < kU; ++u) {
         const float m = vec_max(v[u], T());
         const bool gt = m > vbest;
         vbest = fmax_nan(vbest, m);
@@ -244,6 +245,82 @@ __global__ void ASD_VERIFY_BOUNDS verify_kernel(const VerifyParams p) {
   }
 }
 
+// ---------------------------------------------------------------- one CTA per request (small inputs)
+//
+// When a request's K+1 rows are a few KB, what the streaming kernels pay for is
+// their global round trips (row keys, counters, fences), not the bytes. Here a
+// CTA takes one request: its warps split the request's rows flatly (one round
+// of loads, every lane with up to kSmallUnroll vectors in flight), merge the
+// row keys and the draft logits in shared memory, and warp 0 runs Alg. 1 from
+// there. The workspace is not touched.
+
+constexpr int kSmallThreads = 512;
+constexpr int kSmallUnroll = 8;
+constexpr long long kSmallMaxRequestBytes = 16LL * kSmallThreads * kSmallUnroll;  // 64 KB: one round of loads
+
+template <typename T, bool kStrict>
+__global__ void __launch_bounds__(kSmallThreads) verify_small_kernel(const __grid_constant__ VerifyParams p) {
+  __shared__ unsigned long long s_key[32];
+  __shared__ float s_zx[32];
+  __shared__ unsigned int s_flags;
+  constexpr int VN = Elem<T>::kVec;
+  constexpr int kWarps = kSmallThreads / 32;
+  const int b = blockIdx.x;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int V = p.V, K = p.K, K1 = p.K + 1;
+  if (threadIdx.x < 32) {
+    s_key[threadIdx.x] = 0ull;
+    s_zx[threadIdx.x] = 0.0f;
+  }
+  if (threadIdx.x == 0) s_flags = 0u;
+  float budget = 0.0f, spent = 0.0f;
+  if (!kStrict && threadIdx.x == 0) {  // in flight while the logits stream
+    budget = p.ledger[b].budget;
+    spent = p.ledger[b].spent;
+  }
+  __syncthreads();
+
+  const T* z = static_cast<const T*>(p.logits);
+  const long long n = static_cast<long long>(K1) * V;
+  const long long base = static_cast<long long>(b) * n;
+  long long per = (n + kWarps - 1) / kWarps;
+  per = (per + VN - 1) / VN * VN;
+  const long long lo = base + (warp * per < n ? warp * per : n);
+  const long long hi = base + ((warp + 1) * per < n ? (warp + 1) * per : n);
+  for (long long s0 = lo; s0 < hi;) {
+    const long long row = s0 / V;
+    const long long row0 = row * V;
+    const long long s1 = hi < row0 + V ? hi : row0 + V;
+    const int j = static_cast<int>(row - static_cast<long long>(b) * K1);
+    bool nan = false;
+    const unsigned long long key = segment_key<T, kSmallUnroll>(z, s0, s1, row0, p.head, lane, &nan);
+    if (lane == 0) {
+      atomicMax(&s_key[j], key);
+      if (nan) atomicOr(&s_flags, ASD_STATUS_NAN_LOGIT);
+      if (j < K) {
+        const int x = __ldg(p.draft + static_cast<long long>(b) * K + j);
+        if (x >= 0 && x < V && row0 + x >= s0 && row0 + x < s1) s_zx[j] = Elem<T>::load(z, row0 + x);
+      }
+    }
+    s0 = s1;
+  }
+  __syncthreads();
+  if (warp != 0) return;
+
+  BlockInputs in;
+  in.key = lane < K1 ? s_key[lane] : 0ull;
+  in.x = lane < K ? __ldg(p.draft + static_cast<long long>(b) * K + lane) : -1;
+  in.zx = lane < K ? s_zx[lane] : 0.0f;
+  in.flags = s_flags;
+  in.top = ordered_value(static_cast<uint32_t>(in.key >> 32));
+  in.top_exact = false;
+  budget = __shfl_sync(kFull, budget, 0);
+  spent = __shfl_sync(kFull, spent, 0);
+  bool wrote = false;
+  select_block<T, kStrict>(p, b, in, budget, spent, wrote, lane);
+  if (!kStrict && lane == 0 && wrote) p.ledger[b].spent = spent;
+}
+
 // ---------------------------------------------------------------- TMA pipeline kernel
 //
 // One CTA per SM per launch. The CTA owns an equal, 16-byte aligned slice of
@@ -276,6 +353,9 @@ __global__ void ASD_VERIFY_BOUNDS verify_kernel(const VerifyParams p) {
 #endif
 #ifndef ASD_TMA_MIN_BLOCKS
 #define ASD_TMA_MIN_BLOCKS 3  // CTAs per SM the register allocator must leave room for
+#endif
+#ifndef ASD_TMA_LONE_CTAS_PER_SM
+#define ASD_TMA_LONE_CTAS_PER_SM 3  // CTAs per SM of a launch that cannot overlap the previous one
 #endif
 #ifndef ASD_TMA_L2_HINT
 #define ASD_TMA_L2_HINT 1  // evict-first L2 policy on the streamed logits
@@ -573,6 +653,9 @@ __global__ void __launch_bounds__(kTmaThreads, ASD_TMA_MIN_BLOCKS)
   const int nchunks = lo < hi ? static_cast<int>((hi - lo + kChunkElems - 1) / kChunkElems) : 0;
 
   pdl_signal_dependents();
+  // Unless the caller declared the inputs resident, the previous kernel on the
+  // stream may be the one writing them: read nothing before it has completed.
+  if (!p.resident) pdl_wait_prerequisites();
 
   // each consumer's first row is known now: start its draft-id load before the
   // first copy lands
@@ -828,8 +911,14 @@ int launch_tma(VerifyParams& p, cudaStream_t stream) {
       return ASD_ERR_CUDA;
     info->tma_ready[slot].store(true, std::memory_order_release);
   }
+  // Resident inputs: one CTA per SM, so that three consecutive launches share
+  // the SMs (one ramping up, one streaming, one finishing). Otherwise the
+  // launch reads nothing before the previous kernel completes and runs alone,
+  // so it fills every CTA slot of every SM itself.
+  const long long max_cta =
+      p.resident ? info->sms : static_cast<long long>(info->sms) * ASD_TMA_LONE_CTAS_PER_SM;
   long long ncta = (bulk + kMinPerCta - 1) / kMinPerCta;
-  if (ncta > info->sms) ncta = info->sms;
+  if (ncta > max_cta) ncta = max_cta;
   if (ncta < 1) ncta = 1;
   long long per_cta = (bulk + ncta - 1) / ncta;
   per_cta = (per_cta + VN - 1) / VN * VN;
@@ -868,26 +957,43 @@ int launch_tma(VerifyParams& p, cudaStream_t stream) {
 }
 
 // Which kernel streams the logits: the TMA pipeline for inputs of at least
-// kTmaMinBytes, the register-streaming kernel below that (fewer, shorter
-// warps start faster on tiny inputs). ASD_VERIFY_KERNEL=stream|tma in the
-// environment overrides the choice (used by the tests to cover both kernels).
+// kTmaMinBytes; below that, one CTA per request when a request fits one round
+// of loads of a CTA (single blocks, no vocabulary shard), else the
+// register-streaming kernel (fewer, shorter warps start faster on small
+// inputs). ASD_VERIFY_KERNEL=stream|tma|small in the environment overrides the
+// choice (the tests use it to cover every kernel); `small` falls back to the
+// default when the shape does not qualify.
 constexpr long long kTmaMinBytes = 1LL << 20;
 
-bool use_tma(long long bytes) {
+enum class Path { kSmall, kStream, kTma };
+
+Path choose_path(long long bytes, long long request_bytes, int K, bool single_block) {
+  const bool small_ok = single_block && K + 1 <= 32 && request_bytes <= kSmallMaxRequestBytes;
   const char* env = getenv("ASD_VERIFY_KERNEL");
-  if (env && env[0] == 't') return true;
-  if (env && env[0] == 's') return false;
-  return bytes >= kTmaMinBytes;
+  if (env && strcmp(env, "tma") == 0) return Path::kTma;
+  if (env && strcmp(env, "stream") == 0) return Path::kStream;
+  if (env && strcmp(env, "small") == 0 && small_ok) return Path::kSmall;
+  if (bytes >= kTmaMinBytes) return Path::kTma;
+  return small_ok ? Path::kSmall : Path::kStream;
 }
 
 template <typename T, bool kStrict>
 int launch(VerifyParams& p, cudaStream_t stream) {
-  if (use_tma(p.total * static_cast<long long>(sizeof(T)))) return launch_tma<T, kStrict>(p, stream);
+  const long long request_bytes = static_cast<long long>(p.K + 1) * p.V * static_cast<long long>(sizeof(T));
+  const Path path = choose_path(p.total * static_cast<long long>(sizeof(T)), request_bytes, p.K,
+                                p.nblk == 1 && !p.partials);
+  if (path == Path::kTma) return launch_tma<T, kStrict>(p, stream);
   constexpr int VN = Elem<T>::kVec;
   const uintptr_t addr = reinterpret_cast<uintptr_t>(p.logits);
   if (addr % sizeof(T) != 0) return ASD_ERR_ALIGN;
   long long head = static_cast<long long>(((16 - addr % 16) % 16) / sizeof(T));
   if (head > p.total) head = p.total;
+  if (path == Path::kSmall) {
+    p.head = head;
+    p.per_warp = 0;
+    verify_small_kernel<T, kStrict><<<static_cast<unsigned>(p.B), kSmallThreads, 0, stream>>>(p);
+    return cudaGetLastError() == cudaSuccess ? ASD_OK : ASD_ERR_CUDA;
+  }
   const long long rest = p.total - head;
   int max_warps = 0;
   const int rc = resident_warps<T, kStrict>(&max_warps);
@@ -913,6 +1019,8 @@ int verify_common(bool strict, const void* logits, int dtype, int B, int K, int 
                   int32_t* row_argmax, float* row_regret, int32_t* status, void* workspace,
                   size_t workspace_bytes, cudaStream_t stream, int nblk = 1, int v_offset = 0,
                   int v_total = 0, asd_partial* partials = nullptr) {
+  const bool resident = (dtype & ASD_RESIDENT_INPUTS) != 0;
+  dtype = dtype_code(dtype);
   int rc = check_shape(B, K, V, dtype);
   if (rc != ASD_OK) return rc;
   if (nblk < 0 || (nblk > 0 && B > INT32_MAX / nblk)) return ASD_ERR_SHAPE;
@@ -957,6 +1065,7 @@ int verify_common(bool strict, const void* logits, int dtype, int B, int K, int 
   p.flags = reinterpret_cast<unsigned int*>(ws + l.flags);
   p.error = reinterpret_cast<unsigned int*>(ws + l.error);
   p.row_top = nullptr;
+  p.resident = resident ? 1 : 0;
 
   if (dtype == ASD_F32)
     return strict ? launch<float, true>(p, stream) : launch<float, false>(p, stream);
@@ -1026,8 +1135,9 @@ int asd_verify_launches(int B, int K, int V, int dtype, int* launches) {
   if (!launches) return ASD_ERR_NULL;
   const int rc = check_shape(B, K, V, dtype);
   if (rc != ASD_OK) return rc;
-  const long long bytes = static_cast<long long>(B) * (K + 1) * V * (dtype == ASD_BF16 ? 2 : 4);
-  *launches = B == 0 ? 0 : (use_tma(bytes) && use_split() ? 2 : 1);
+  const long long request_bytes = static_cast<long long>(K + 1) * V * (dtype_code(dtype) == ASD_BF16 ? 2 : 4);
+  const Path path = choose_path(request_bytes * B, request_bytes, K, true);
+  *launches = B == 0 ? 0 : (path == Path::kTma && use_split() ? 2 : 1);
   return ASD_OK;
 }
 

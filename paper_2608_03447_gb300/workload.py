@@ -20,8 +20,10 @@ def l2_bytes(device=None) -> int:
 class VerifyWorkload:
     def __init__(self, B: int, K: int, V: int, dtype: torch.dtype, gate: float, cap: int, budget: float,
                  config: int = 1, nbuf: int | None = None, min_total_bytes: int | None = None,
-                 mix=inputs.MIX_DEFAULT, device="cuda", with_rows: bool = False, strict: bool = False):
+                 mix=inputs.MIX_DEFAULT, device="cuda", with_rows: bool = False, strict: bool = False,
+                 resident: bool = False):
         self.B, self.K, self.V, self.dtype = B, K, V, dtype
+        self.resident = resident  # pass ASD_RESIDENT_INPUTS: the buffers are written once, before any step
         self.gate, self.cap, self.budget, self.strict = gate, cap, budget, strict
         self.device = torch.device(device)
         elem = torch.tensor([], dtype=dtype).element_size()
@@ -47,9 +49,10 @@ class VerifyWorkload:
     def step(self, i: int, stream=None) -> dict:
         k = i % self.nbuf
         if self.strict:
-            return asd.verify_strict(self.logits[k], self.drafts[k], self.workspace, self.out, stream)
+            return asd.verify_strict(self.logits[k], self.drafts[k], self.workspace, self.out, stream,
+                                     resident=self.resident)
         return asd.verify(self.logits[k], self.drafts[k], self.ledger, self.gate, self.cap,
-                          self.workspace, self.out, stream)
+                          self.workspace, self.out, stream, resident=self.resident)
 
     def capture(self, nsteps: int, first: int = 0) -> torch.cuda.CUDAGraph:
         """Capture steps first .. first+nsteps-1 into one CUDA graph (one kernel node per step)."""

@@ -19,9 +19,10 @@ pytestmark = pytest.mark.gpu
 INT32_MAX = 2**31 - 1
 
 
-@pytest.fixture(params=["stream", "tma"])
+@pytest.fixture(params=["stream", "tma", "small"])
 def kernel(request, monkeypatch):
-    """Runs the test through the register-streaming kernel and through the TMA pipeline kernel."""
+    """Runs the test through the register-streaming kernel, the TMA pipeline kernel and the
+    one-CTA-per-request kernel (shapes it does not take fall back to the default choice)."""
     monkeypatch.setenv("ASD_VERIFY_KERNEL", request.param)
     return request.param
 
@@ -30,11 +31,11 @@ def _np(out: dict) -> dict:
     return {k: v.cpu().numpy() for k, v in out.items()}
 
 
-def gpu_verify(asd, logits, draft, ledger, gate, cap, strict=False):
+def gpu_verify(asd, logits, draft, ledger, gate, cap, strict=False, resident=False):
     if strict:
-        out = asd.verify_strict(logits, draft)
+        out = asd.verify_strict(logits, draft, resident=resident)
     else:
-        out = asd.verify(logits, draft, ledger, gate, cap)
+        out = asd.verify(logits, draft, ledger, gate, cap, resident=resident)
     torch.cuda.synchronize()
     res = _np(out)
     if ledger is not None:
@@ -61,18 +62,19 @@ def assert_parity(gpu: dict, orc: dict, what: str = "", ledger: bool = True):
         assert np.array_equal(gpu["ledger"].view(np.uint32), orc["ledger"].view(np.uint32)), f"{what}: ledger"
 
 
-def run_sequence(asd, B, K, V, dtype, blocks, gate, cap, budget, config, mix=inputs.MIX_DEFAULT, point=0):
+def run_sequence(asd, B, K, V, dtype, blocks, gate, cap, budget, config, mix=inputs.MIX_DEFAULT, point=0,
+                 resident=False):
     """Sequential blocks on the same requests; the GPU carries its ledger on the device."""
     led_gpu = asd.make_ledger(B, budget)
     led_orc = np.array([[budget, 0.0]] * B, np.float32)
     for blk in blocks:
         b = inputs.gen_block(B, K, V, dtype, inputs.seed_for(config, point, blk), "cuda", mix=mix)
-        g = gpu_verify(asd, b.logits, b.draft, led_gpu, gate, cap)
+        g = gpu_verify(asd, b.logits, b.draft, led_gpu, gate, cap, resident=resident)
         o = oracle.verify(b.logits.cpu(), b.draft.cpu().numpy(), led_orc, gate, cap)
         assert_parity(g, o, f"config {config} block {blk}")
         led_orc = o["ledger"]
         # strict entry on the same block
-        gs = gpu_verify(asd, b.logits, b.draft, None, 0, 0, strict=True)
+        gs = gpu_verify(asd, b.logits, b.draft, None, 0, 0, strict=True, resident=resident)
         os_ = oracle.verify(b.logits.cpu(), b.draft.cpu().numpy(), None, strict=True)
         assert_parity(gs, os_, f"config {config} block {blk} strict", ledger=False)
     return led_orc
@@ -98,10 +100,11 @@ def test_tiny_zero_budget_is_strict(asd, kernel):
         assert np.array_equal(g["ledger"], np.zeros((B, 2), np.float32))
 
 
-def test_qwen3_shape_bf16_blocks(asd, kernel):
+@pytest.mark.parametrize("resident", [False, True])
+def test_qwen3_shape_bf16_blocks(asd, kernel, resident):
     cfg = inputs.CONFIGS[1]
     run_sequence(asd, cfg["B"], cfg["K"], cfg["V"], cfg["dtype"], range(8), cfg["gate"], cfg["cap"],
-                 cfg["budget"], 1)
+                 cfg["budget"], 1, resident=resident)
 
 
 def test_budget_cap_sweep(asd):
@@ -337,3 +340,47 @@ def test_bounded_wait_reports_timeout_and_context_survives(asd):
     assert np.array_equal(out["accepted_len"].cpu().numpy(), o["accepted_len"])
     assert np.array_equal(out["committed"].cpu().numpy(), o["committed"])
     assert np.array_equal(led.cpu().numpy().view(np.int32), o["ledger"].view(np.int32))
+
+
+@pytest.mark.parametrize("shape", [(32, 8, 151936), (4, 8, 1024)])
+def test_logits_written_by_the_previous_kernel(asd, shape):
+    """Without ASD_RESIDENT_INPUTS the logits may come from the kernel right before the call on the same
+    stream (as from the model's LM head): every call sees that kernel's output, eagerly and in a CUDA graph."""
+    B, K, V = shape
+    blocks = [inputs.gen_block(B, K, V, torch.bfloat16, 8800 + i, "cuda") for i in range(4)]
+    expect = [oracle.verify(b.logits.cpu(), b.draft.cpu().numpy(), np.array([[8.0, 0.0]] * B, np.float32), 1.0, 2)
+              for b in blocks]
+    buf = torch.empty_like(blocks[0].logits)
+    ledgers = [asd.make_ledger(B, 8.0) for _ in range(8)]
+    outs = [asd.alloc_outputs(B, K) for _ in range(8)]
+    ws = asd.Workspace(B, K, V, asd.BF16)
+
+    def sequence():
+        for n in range(8):
+            b = blocks[n % 4]
+            torch.mul(b.logits, 1, out=buf)  # a kernel writes the logits; the verify follows it directly
+            asd.verify(buf, b.draft, ledgers[n], 1.0, 2, workspace=ws, out=outs[n])
+
+    def check(what):
+        torch.cuda.synchronize()
+        for n in range(8):
+            o, g = expect[n % 4], _np(outs[n])
+            for key in ("accepted_len", "committed", "recovery", "row_argmax", "status"):
+                assert np.array_equal(g[key], o[key]), f"{what} call {n}: {key}"
+            assert np.array_equal(ledgers[n].cpu().numpy().view(np.int32), o["ledger"].view(np.int32))
+
+    for _ in range(3):
+        for led in ledgers:
+            led.copy_(asd.make_ledger(B, 8.0))
+        sequence()
+        check("eager")
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=side):
+        sequence()
+    for _ in range(3):
+        for led in ledgers:
+            led.copy_(asd.make_ledger(B, 8.0))
+        graph.replay()
+        check("graph")
