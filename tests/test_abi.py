@@ -46,6 +46,25 @@ def test_workspace_size(lib):
     assert lib.asd_workspace_size(1, 4, 10, asd.F32, None) == 1
 
 
+def test_resident_inputs_flag_is_a_flag_not_a_dtype(lib):
+    """ASD_RESIDENT_INPUTS rides in the dtype argument: it changes no size or validation, and any other
+    high bit is still an unknown dtype."""
+    sz, sz_flag = ctypes.c_size_t(0), ctypes.c_size_t(0)
+    for dt in (asd.F32, asd.BF16):
+        assert lib.asd_workspace_size(8, 4, 1000, dt, ctypes.byref(sz)) == 0
+        assert lib.asd_workspace_size(8, 4, 1000, dt | asd.RESIDENT_INPUTS, ctypes.byref(sz_flag)) == 0
+        assert sz.value == sz_flag.value
+        n, n_flag = ctypes.c_int(0), ctypes.c_int(0)
+        for (B, K, V) in ((32, 8, 151936), (4, 8, 1024)):
+            assert lib.asd_verify_launches(B, K, V, dt, ctypes.byref(n)) == 0
+            assert lib.asd_verify_launches(B, K, V, dt | asd.RESIDENT_INPUTS, ctypes.byref(n_flag)) == 0
+            assert n.value == n_flag.value
+    assert lib.asd_workspace_size(8, 4, 1000, asd.F32 | 0x200, ctypes.byref(sz)) == 3
+    assert _verify(lib, dtype=asd.F32 | 0x200) == 3
+    assert _verify(lib, dtype=asd.F32 | asd.RESIDENT_INPUTS, B=0) == 0
+    assert _verify(lib, dtype=asd.BF16 | asd.RESIDENT_INPUTS, K=32) == 2
+
+
 def _verify(lib, **kw):
     a = dict(logits=0x1000, dtype=asd.F32, B=2, K=3, V=10, draft=0x2000, ledger=0x3000, gate=1.0, cap=2,
              acc=0x4000, com=0x5000, rec=0x6000, ya=NULL, rr=NULL, st=NULL, ws=0x7000, wsb=1 << 20)
