@@ -278,9 +278,25 @@ def cpu_baseline(wl, seconds: float = 12.0) -> dict:
             if time.perf_counter() - t0 >= seconds:
                 break
     dt = time.perf_counter() - t0
+    # one thread, and the two stages apart: the row stage (the strict oracle: argmax, draft logits,
+    # regrets, plus Eq. 2's trivial selection) and Alg. 1 alone (oracle_select on those rows)
+    z, x = host[0]
+    n1, t1 = 0, time.perf_counter()
+    while time.perf_counter() - t1 < 2.0:
+        rows_out = oracle.verify(z, x, None, strict=True, dtype=oracle.DTYPE_BF16, lib=lib)
+        n1 += 1
+    row_ms = (time.perf_counter() - t1) / n1 * 1e3
+    n2, t2 = 0, time.perf_counter()
+    while time.perf_counter() - t2 < 0.5:
+        oracle.select(x, rows_out["row_argmax"], rows_out["row_regret"], rows_out["status"], led, GATE, CAP, lib=lib)
+        n2 += 1
+    sel_ms = (time.perf_counter() - t2) / n2 * 1e3
     return {"value": rows / dt, "unit": "rows/s", "cores": cores, "kind": "oracle",
             "sample": f"{i} full blocks ({B}x{K + 1}x{V} bf16 from the GPU buffers), one request per thread, "
-                      f"{dt:.1f} s"}
+                      f"{dt:.1f} s",
+            "single_thread": {"rows_per_s": B * (K + 1) / ((row_ms + sel_ms) / 1e3),
+                              "row_stage_ms_per_block": row_ms, "selection_ms_per_block": sel_ms,
+                              "sample": f"{n1} row-stage and {n2} selection passes over one block"}}
 
 
 def run_gpu(args) -> None:
