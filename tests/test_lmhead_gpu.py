@@ -98,8 +98,11 @@ def compare(out, z64, z32, draft, tokens, B, K, gate, cap, budget):
     return n_eligible, len(reqs)
 
 
-@pytest.mark.parametrize("T,H,V", [(36, 512, 1000), (300, 136, 777), (130, 64, 256), (129, 5120, 2100)])
+@pytest.mark.parametrize("T,H,V", [(36, 512, 1000), (300, 136, 777), (130, 64, 256), (129, 5120, 2100),
+                                   (5, 64, 1), (200, 72, 257), (15000, 64, 300)])
 def test_lmhead_logits_match_fp64(asd, T, H, V):
+    """Includes V = 1, a last 256-row vocabulary tile holding one row, and more token tiles (79) than
+    SM pairs, so the grid runs in two waves."""
     g = torch.Generator(device="cuda").manual_seed(T * 7 + H + V)
     h = torch.randn(T, H, generator=g, device="cuda").to(torch.bfloat16)
     w = (0.02 * torch.randn(V, H, generator=g, device="cuda")).to(torch.bfloat16)
@@ -159,7 +162,8 @@ def test_lmhead_full_size_sampled(asd):
     assert n_ok >= 1
 
 
-@pytest.mark.parametrize("B,K,H,V", [(8, 8, 512, 1000), (40, 8, 256, 2100), (5, 0, 64, 777), (3, 16, 320, 1300)])
+@pytest.mark.parametrize("B,K,H,V", [(8, 8, 512, 1000), (40, 8, 256, 2100), (5, 0, 64, 777), (3, 16, 320, 1300),
+                                     (1500, 9, 64, 300)])
 def test_lmhead_verify_exact_inputs_bit_exact(asd, B, K, H, V):
     """Integer h and W: the fp32 logits are exact, so every output equals the oracle's bit for bit,
     ties across warps, SMs and SM pairs included (lowest index wins)."""
