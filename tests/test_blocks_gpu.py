@@ -16,9 +16,11 @@ from paper_2608_03447_gb300 import inputs
 pytestmark = pytest.mark.gpu
 
 
-@pytest.fixture(params=["stream", "tma"])
+@pytest.fixture(params=["stream", "tma", "tma-fused"])
 def kernel(request, monkeypatch):
-    monkeypatch.setenv("ASD_VERIFY_KERNEL", request.param)
+    """tma-fused: the TMA row stage with the selection inside it (ASD_VERIFY_SPLIT=0)."""
+    monkeypatch.setenv("ASD_VERIFY_KERNEL", request.param.split("-")[0])
+    monkeypatch.setenv("ASD_VERIFY_SPLIT", "0" if request.param.endswith("fused") else "1")
     return request.param
 
 

@@ -19,11 +19,13 @@ pytestmark = pytest.mark.gpu
 INT32_MAX = 2**31 - 1
 
 
-@pytest.fixture(params=["stream", "tma", "small"])
+@pytest.fixture(params=["stream", "tma", "tma-fused", "small"])
 def kernel(request, monkeypatch):
-    """Runs the test through the register-streaming kernel, the TMA pipeline kernel and the
-    one-CTA-per-request kernel (shapes it does not take fall back to the default choice)."""
-    monkeypatch.setenv("ASD_VERIFY_KERNEL", request.param)
+    """Runs the test through the register-streaming kernel, the TMA pipeline kernel (with its selection
+    kernel, and with the selection inside the row stage: ASD_VERIFY_SPLIT=0) and the one-CTA-per-request
+    kernel (shapes it does not take fall back to the default choice)."""
+    monkeypatch.setenv("ASD_VERIFY_KERNEL", request.param.split("-")[0])
+    monkeypatch.setenv("ASD_VERIFY_SPLIT", "0" if request.param.endswith("fused") else "1")
     return request.param
 
 
