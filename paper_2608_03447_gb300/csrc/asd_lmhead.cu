@@ -113,24 +113,30 @@ __device__ __forceinline__ void cluster_sync_all() {
 __device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr) {
   asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
 }
+// One bounded wait on the phase with the given parity. The thread may sleep
+// until the phase completes (at most kSuspendNs per call), so the warps that
+// wait -- most of them, most of the time -- take no issue slots from the MMA
+// and TMA threads (polling them cost this kernel about 7 %).
+constexpr uint32_t kSuspendNs = 1000000;
 __device__ __forceinline__ bool mbar_try_wait_cluster(unsigned long long* bar, uint32_t parity) {
   uint32_t done;
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(done)
-      : "r"(smem_u32(bar)), "r"(parity)
+      : "r"(smem_u32(bar)), "r"(parity), "r"(kSuspendNs)
       : "memory");
   return done != 0;
 }
-// mbar_wait for barriers that the other CTA of the pair also signals.
+// mbar_wait for barriers that the other CTA of the pair also signals; the
+// abort flag and the clock are checked every 16 sleeps.
 __device__ inline bool mbar_wait_cluster(unsigned long long* bar, uint32_t parity, volatile int* abort) {
   if (mbar_try_wait_cluster(bar, parity)) return true;
   const unsigned long long t0 = global_ns();
   for (unsigned it = 1;; ++it) {
     if (mbar_try_wait_cluster(bar, parity)) return true;
-    if ((it & 255u) == 0) {
+    if ((it & 15u) == 0) {
       if (*abort) return false;
       if (global_ns() - t0 > kWaitLimitNs) return false;
     }
