@@ -273,8 +273,14 @@ __global__ void __launch_bounds__(kSmallThreads) verify_small_kernel(const __gri
     s_zx[threadIdx.x] = 0.0f;
   }
   if (threadIdx.x == 0) s_flags = 0u;
+  // Programmatic dependent launch: the next call's CTAs may start now. With
+  // resident inputs this call reads its logits and drafts before the previous
+  // kernel on the stream has completed; the ledger and the outputs, which that
+  // kernel may use, wait for it in every case.
+  pdl_signal_dependents();
+  if (!p.resident) pdl_wait_prerequisites();
   float budget = 0.0f, spent = 0.0f;
-  if (!kStrict && threadIdx.x == 0) {  // in flight while the logits stream
+  if (!kStrict && !p.resident && threadIdx.x == 0) {  // in flight while the logits stream
     budget = p.ledger[b].budget;
     spent = p.ledger[b].spent;
   }
@@ -306,6 +312,13 @@ __global__ void __launch_bounds__(kSmallThreads) verify_small_kernel(const __gri
   }
   __syncthreads();
   if (warp != 0) return;
+  if (p.resident) {
+    pdl_wait_prerequisites();
+    if (!kStrict && lane == 0) {
+      budget = p.ledger[b].budget;
+      spent = p.ledger[b].spent;
+    }
+  }
 
   BlockInputs in;
   in.key = lane < K1 ? s_key[lane] : 0ull;
@@ -991,7 +1004,19 @@ int launch(VerifyParams& p, cudaStream_t stream) {
   if (path == Path::kSmall) {
     p.head = head;
     p.per_warp = 0;
-    verify_small_kernel<T, kStrict><<<static_cast<unsigned>(p.B), kSmallThreads, 0, stream>>>(p);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(p.B));
+    cfg.blockDim = dim3(kSmallThreads);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    const char* env = getenv("ASD_VERIFY_PDL");
+    if (!(env && env[0] == '0')) {
+      cfg.attrs = attr;
+      cfg.numAttrs = 1;
+    }
+    if (cudaLaunchKernelEx(&cfg, verify_small_kernel<T, kStrict>, p) != cudaSuccess) return ASD_ERR_CUDA;
     return cudaGetLastError() == cudaSuccess ? ASD_OK : ASD_ERR_CUDA;
   }
   const long long rest = p.total - head;

@@ -82,10 +82,13 @@ def run_sequence(asd, B, K, V, dtype, blocks, gate, cap, budget, config, mix=inp
     return led_orc
 
 
-def test_tiny_fp32_sixteen_blocks(asd, kernel):
+@pytest.mark.parametrize("resident", [False, True])
+def test_tiny_fp32_sixteen_blocks(asd, kernel, resident):
+    """Sixteen dependent calls (each reads the ledger the previous one wrote), with and without
+    ASD_RESIDENT_INPUTS: the early start of a call never reads the ledger early."""
     cfg = inputs.CONFIGS[0]
     led = run_sequence(asd, cfg["B"], cfg["K"], cfg["V"], cfg["dtype"], range(cfg["blocks"]),
-                       cfg["gate"], cfg["cap"], cfg["budget"], 0)
+                       cfg["gate"], cfg["cap"], cfg["budget"], 0, resident=resident)
     assert np.all(led[:, 1] <= cfg["budget"])
 
 
@@ -384,5 +387,51 @@ def test_logits_written_by_the_previous_kernel(asd, shape):
     for _ in range(3):
         for led in ledgers:
             led.copy_(asd.make_ledger(B, 8.0))
+        graph.replay()
+        check("graph")
+
+
+@pytest.mark.parametrize("resident", [False, True])
+@pytest.mark.parametrize("shape", [(4, 8, 1024, torch.float32, 16), (32, 8, 151936, torch.bfloat16, 6)])
+def test_back_to_back_calls_carry_the_ledger(asd, shape, resident):
+    """Dependent calls issued back to back with no synchronisation in between (eagerly and as one
+    CUDA graph): each reads the ledger the previous one wrote, which a call that starts early
+    (programmatic dependent launch) must not read before that call has completed."""
+    B, K, V, dtype, n = shape
+    blocks = [inputs.gen_block(B, K, V, dtype, 9100 + i, "cuda") for i in range(n)]
+    led0 = np.array([[4.0, 0.0]] * B, np.float32)
+    expect, led = [], led0
+    for b in blocks:
+        o = oracle.verify(b.logits.cpu(), b.draft.cpu().numpy(), led, 1.0, 2)
+        expect.append(o)
+        led = o["ledger"]
+    ledger = torch.from_numpy(led0).cuda()
+    outs = [asd.alloc_outputs(B, K) for _ in range(n)]
+    ws = asd.Workspace(B, K, V, asd.BF16 if dtype == torch.bfloat16 else asd.F32)
+
+    def sequence():
+        for i, b in enumerate(blocks):
+            asd.verify(b.logits, b.draft, ledger, 1.0, 2, workspace=ws, out=outs[i], resident=resident)
+
+    def check(what):
+        torch.cuda.synchronize()
+        for i in range(n):
+            g = _np(outs[i])
+            for key in ("accepted_len", "committed", "recovery", "row_argmax", "status"):
+                assert np.array_equal(g[key], expect[i][key]), f"{what} call {i}: {key}"
+            assert np.array_equal(g["row_regret"].view(np.int32), expect[i]["row_regret"].view(np.int32))
+        assert np.array_equal(ledger.cpu().numpy().view(np.int32), expect[-1]["ledger"].view(np.int32))
+
+    sequence()
+    check("eager")
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    graph = torch.cuda.CUDAGraph()
+    ledger.copy_(torch.from_numpy(led0))
+    torch.cuda.synchronize()
+    with torch.cuda.graph(graph, stream=side):
+        sequence()
+    for _ in range(2):
+        ledger.copy_(torch.from_numpy(led0).cuda())
         graph.replay()
         check("graph")
