@@ -284,13 +284,18 @@ def verify_strict(logits: torch.Tensor, draft: torch.Tensor, workspace: Workspac
 
 
 _aliases: dict = {}
+_ALIAS_CACHE = 64  # the most recently used pinned buffers keep their looked-up device address
 
 
 def _alias(t: torch.Tensor) -> int:
     key = (t.data_ptr(), t.numel() * t.element_size())
-    if key not in _aliases:
-        _aliases[key] = host_alias(t)
-    return _aliases[key]
+    addr = _aliases.pop(key, None)
+    if addr is None:
+        addr = host_alias(t)
+    _aliases[key] = addr  # re-inserted: dicts keep insertion order, so the oldest entry is first
+    while len(_aliases) > _ALIAS_CACHE:
+        _aliases.pop(next(iter(_aliases)))
+    return addr
 
 
 def verify_from_host(logits_host: torch.Tensor, draft_host: torch.Tensor, ledger: torch.Tensor, gate: float,
