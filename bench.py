@@ -115,8 +115,30 @@ def run_lmhead(dev, iters: int = 20) -> dict:
     flop = 2.0 * LM_B * (LM_K + 1) * LM_H * LM_V
     tflops = flop / (ms * 1e-3) / 1e12
     pk = bf16_peaks()
+    # one of four tensor-parallel ranks: its quarter of W, the partials (the all-gather and the
+    # combine follow; the combine is timed with the sharded verify row)
+    S = 4
+    vs = LM_V // S
+    shard = inp.weight[:vs].contiguous()
+    parts = torch.empty(LM_B * (LM_K + 1), asd.PARTIAL_WORDS, dtype=torch.int32, device=dev)
+    sws = asd.lmhead_workspace(LM_B, LM_K, vs, LM_H, dev)
+    for _ in range(3):
+        asd.lmhead_partials(inp.hidden, shard, inp.draft, 0, LM_V, workspace=sws, out=parts)
+    torch.cuda.synchronize(dev)
+    s2, e2 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s2.record(stream)
+    for _ in range(iters):
+        asd.lmhead_partials(inp.hidden, shard, inp.draft, 0, LM_V, workspace=sws, out=parts)
+    e2.record(stream)
+    e2.synchronize()
+    ms_rank = s2.elapsed_time(e2) / iters
+    del shard
+    rank_tflops = flop / S / (ms_rank * 1e-3) / 1e12
     return {"workload": LM_WORKLOAD, "ms_per_step": ms, "rows_per_s": LM_B * (LM_K + 1) / (ms * 1e-3),
             "launches": iters,
+            "per_rank_of_4": {"ms": ms_rank, "tflops": rank_tflops, "frac": rank_tflops / pk["burst"],
+                              "workload": f"asd_lmhead_partials on a {vs} x {LM_H} shard of W (one of {S} "
+                                          "tensor-parallel ranks), 576 rows"},
             "roofline": {"bound": "tensor", "achieved": tflops, "peak": pk["burst"], "unit": "TFLOP/s",
                          "frac": tflops / pk["burst"], "peak_kind": "burst (kernel timed alone)",
                          "peak_source": pk["source"], "traffic": recorded_traffic("lmhead_verify_kernel"),

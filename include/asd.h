@@ -297,6 +297,18 @@ int asd_shard_combine(const asd_partial* partials, int S, int B, int K, int V, c
                       int32_t* committed, int32_t* recovery, int32_t* row_argmax, float* row_regret,
                       int32_t* status, asd_stream_t stream);
 
+/* Step 1 of the same scheme with the LM head fused (the remark of Sec. 3.3 as
+ * a tensor-parallel rank would run it: no logit buffer anywhere):
+ * weight [Vs, H] bf16 holds rows v_offset .. v_offset+Vs-1 of the LM-head
+ * weight of a V-entry vocabulary; hidden [B*(K+1), H] bf16 and draft [B, K]
+ * (GLOBAL ids) as in asd_lmhead_verify; writes partials [B*(K+1)] for
+ * asd_shard_combine. The top logit in a partial is the value the key holds
+ * (a zero maximum is +0). Workspace from asd_lmhead_workspace_size(B, K, Vs,
+ * H). Same precision and launch notes as asd_lmhead_verify. */
+int asd_lmhead_partials(const void* hidden, const void* weight, int H, int B, int K, int Vs, int v_offset,
+                        int V, const int32_t* draft, asd_partial* partials, void* workspace,
+                        size_t workspace_bytes, asd_stream_t stream);
+
 /*
  * Advance along the emitted sequence (Sec. 3.3: the target cache, the draft
  * cache and the ledger advance only along the emitted tokens; proposal-only

@@ -88,6 +88,8 @@ def _declare(lib: ctypes.CDLL) -> ctypes.CDLL:
     lib.asd_lmhead_verify.restype = i32
     lib.asd_lmhead_logits.argtypes = [vp, vp, i32, i32, i32, vp, vp]
     lib.asd_lmhead_logits.restype = i32
+    lib.asd_lmhead_partials.argtypes = [vp, vp, i32, i32, i32, i32, i32, i32, vp, vp, vp, sz, vp]
+    lib.asd_lmhead_partials.restype = i32
     return lib
 
 
@@ -361,6 +363,25 @@ def lmhead_verify(hidden: torch.Tensor, weight: torch.Tensor, draft: torch.Tenso
                                   _ptr(o.get("row_argmax")), _ptr(o.get("row_regret")), _ptr(o.get("row_top")),
                                   _ptr(o.get("status")), ws.ptr, ws.nbytes, _stream(stream))
     _check("asd_lmhead_verify", rc)
+    return o
+
+
+def lmhead_partials(hidden: torch.Tensor, weight_shard: torch.Tensor, draft: torch.Tensor, v_offset: int, V: int,
+                    workspace: Workspace | None = None, out: torch.Tensor | None = None,
+                    stream=None) -> torch.Tensor:
+    """asd_lmhead_partials: one vocabulary shard of the fused LM-head verify, as int32 [B*(K+1), 6] partials.
+
+    weight_shard [Vs, H] holds rows v_offset .. v_offset+Vs-1 of the LM-head weight; draft holds global ids.
+    """
+    T, Vs, H = _lm_shapes(hidden, weight_shard)
+    B, K = draft.shape
+    if T != B * (K + 1):
+        raise ValueError("hidden must hold B*(K+1) rows")
+    ws = workspace or lmhead_workspace(B, K, Vs, H, hidden.device, stream)
+    o = out if out is not None else torch.empty(T, PARTIAL_WORDS, dtype=torch.int32, device=hidden.device)
+    _check("asd_lmhead_partials", load().asd_lmhead_partials(_ptr(hidden), _ptr(weight_shard), H, B, K, Vs,
+                                                             int(v_offset), int(V), _ptr(draft), _ptr(o), ws.ptr,
+                                                             ws.nbytes, _stream(stream)))
     return o
 
 

@@ -239,7 +239,7 @@ __device__ void emit_partials(const VerifyParams& p, int b, int lane) {
     const long long row = static_cast<long long>(b) * K1 + lane;
     const uint32_t local = 0xffffffffu - static_cast<uint32_t>(in.key);
     float top = in.top;
-    if (top == 0.0f && in.key) top = Elem<T>::load(z, row * p.V + local);  // keep the sign of a zero
+    if (top == 0.0f && in.key && z) top = Elem<T>::load(z, row * p.V + local);  // keep the sign of a zero
     const int xl = lane < K ? in.x - p.v_offset : -1;
     asd_partial out;
     out.key = in.key ? ((in.key & 0xffffffff00000000ull) |

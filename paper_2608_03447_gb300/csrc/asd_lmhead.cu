@@ -284,7 +284,9 @@ __global__ void __launch_bounds__(kLmThreads, 1)
       const int tok = m * kTN + c;
       int x = -1;
       if (tok < q.T && (tok % K1) < p.K) {
-        x = __ldg(p.draft + static_cast<long long>(tok / K1) * p.K + (tok % K1));
+        // the row of this CTA's weight that holds the draft token (a vocabulary
+        // shard starts at global index v_offset), if any
+        x = __ldg(p.draft + static_cast<long long>(tok / K1) * p.K + (tok % K1)) - p.v_offset;
         if (x < 0 || x >= p.V) x = -1;
       }
       sh.draft[c] = x;
@@ -677,6 +679,41 @@ int asd_lmhead_verify(const void* hidden, const void* weight, int H, int B, int 
   p.nblk = 1;
   return launch_lmhead<false, false>(hidden, weight, H, B * (K + 1), p, nullptr,
                                      reinterpret_cast<cudaStream_t>(stream));
+}
+
+int asd_lmhead_partials(const void* hidden, const void* weight, int H, int B, int K, int Vs, int v_offset,
+                        int V, const int32_t* draft, asd_partial* partials, void* workspace,
+                        size_t workspace_bytes, asd_stream_t stream) {
+  int rc = check_shape(B, K, Vs, ASD_BF16);
+  if (rc != ASD_OK) return rc;
+  if (v_offset < 0 || V < 1 || static_cast<long long>(v_offset) + Vs > V) return ASD_ERR_SHAPE;
+  if (B == 0) return ASD_OK;
+  rc = check_lm_inputs(hidden, weight, H);
+  if (rc != ASD_OK) return rc;
+  if (!partials || !workspace) return ASD_ERR_NULL;
+  if (K > 0 && !draft) return ASD_ERR_NULL;
+  const WorkspaceLayout l = layout_for(B, K);
+  if (workspace_bytes < l.total) return ASD_ERR_WORKSPACE;
+  if (reinterpret_cast<uintptr_t>(workspace) % 16 != 0) return ASD_ERR_ALIGN;
+  char* ws = static_cast<char*>(workspace);
+  VerifyParams p = {};
+  p.logits = nullptr;
+  p.B = B;
+  p.K = K;
+  p.V = Vs;
+  p.total = static_cast<long long>(B) * (K + 1);
+  p.draft = draft;
+  p.row_key = reinterpret_cast<unsigned long long*>(ws + l.row_key);
+  p.draft_logit = reinterpret_cast<float*>(ws + l.draft_logit);
+  p.done = reinterpret_cast<unsigned long long*>(ws + l.done);
+  p.flags = reinterpret_cast<unsigned int*>(ws + l.flags);
+  p.error = reinterpret_cast<unsigned int*>(ws + l.error);
+  p.nblk = 1;
+  p.v_offset = v_offset;
+  p.v_total = V;
+  p.partials = partials;
+  return launch_lmhead<true, false>(hidden, weight, H, B * (K + 1), p, nullptr,
+                                    reinterpret_cast<cudaStream_t>(stream));
 }
 
 int asd_lmhead_logits(const void* hidden, const void* weight, int H, int T, int V, float* logits,

@@ -214,3 +214,36 @@ def test_lmhead_verify_nan_row_flags_its_request(asd):
         assert out["accepted_len"][b].item() == o["accepted_len"][b]
         assert np.array_equal(out["committed"][b].cpu().numpy(), o["committed"][b])
         assert np.array_equal(led.cpu().numpy()[b].view(np.int32), o["ledger"][b].view(np.int32))
+
+
+@pytest.mark.parametrize("B,K,H,V,bounds", [(8, 8, 256, 1000, (0, 300, 650, 1000)),
+                                            (40, 8, 128, 2100, (0, 512, 1000, 1601, 2100)),
+                                            (5, 0, 64, 777, (0, 129, 777)),
+                                            (3, 16, 320, 1300, (0, 1, 1300))])
+def test_lmhead_sharded_partials_combine_to_the_unsharded_verify(asd, B, K, H, V, bounds):
+    """The fused LM-head per vocabulary shard (a tensor-parallel rank's share of W), its partials
+    combined: every output equals the unsharded fused verify and the oracle, bit for bit (exact
+    inputs), with shard edges inside 256-row tiles, a one-row shard, and ties across shards."""
+    inp = inputs.gen_lmhead_exact(B, K, H, V, 7300 + B + K + H, "cuda")
+    T = B * (K + 1)
+    S = len(bounds) - 1
+    parts = torch.empty(S, T, asd.PARTIAL_WORDS, dtype=torch.int32, device="cuda")
+    for i in range(S):
+        shard = inp.weight[bounds[i]:bounds[i + 1]].contiguous()
+        asd.lmhead_partials(inp.hidden, shard, inp.draft, bounds[i], V, out=parts[i])
+    led_s = asd.make_ledger(B, 8.0)
+    sharded = asd.shard_combine(parts, inp.draft, led_s, 1.0, 2, V)
+    led_u = asd.make_ledger(B, 8.0)
+    whole = asd.lmhead_verify(inp.hidden, inp.weight, inp.draft, led_u, 1.0, 2)
+    torch.cuda.synchronize()
+    for key in ("accepted_len", "committed", "recovery", "row_argmax", "status"):
+        assert np.array_equal(sharded[key].cpu().numpy(), whole[key].cpu().numpy()), key
+    assert np.array_equal(sharded["row_regret"].cpu().numpy().view(np.int32),
+                          whole["row_regret"].cpu().numpy().view(np.int32))
+    assert np.array_equal(led_s.cpu().numpy().view(np.int32), led_u.cpu().numpy().view(np.int32))
+    z64, z32 = oracle_logits(inp.hidden, inp.weight, range(T))
+    o = oracle.verify(z32.reshape(B, K + 1, V), inp.draft.cpu().numpy(), np.array([[8.0, 0.0]] * B, np.float32),
+                      1.0, 2)
+    for key in ("accepted_len", "committed", "recovery", "row_argmax", "status"):
+        assert np.array_equal(sharded[key].cpu().numpy(), o[key]), f"oracle: {key}"
+    assert np.array_equal(led_s.cpu().numpy().view(np.int32), o["ledger"].view(np.int32))
