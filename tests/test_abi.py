@@ -107,6 +107,32 @@ def test_strict_rejects_bad_arguments(lib):
     assert strict(wsb=0) == 5
 
 
+def test_lmhead_entry_points_reject_bad_arguments(lib):
+    """The fused LM-head entry points validate shapes, pointers and alignment before any CUDA call."""
+    sz = ctypes.c_size_t(0)
+    assert lib.asd_lmhead_workspace_size(4, 8, 1000, 64, ctypes.byref(sz)) == 0 and sz.value > 0
+    assert lib.asd_lmhead_workspace_size(4, 8, 1000, 60, ctypes.byref(sz)) == 2   # H not a multiple of 8
+
+    def partials(**kw):
+        a = dict(h=0x1000, w=0x2000, H=64, B=2, K=3, Vs=100, off=0, V=400, draft=0x3000, out=0x4000,
+                 ws=0x7000, wsb=1 << 20)
+        a.update(kw)
+        return lib.asd_lmhead_partials(a["h"], a["w"], a["H"], a["B"], a["K"], a["Vs"], a["off"], a["V"],
+                                       a["draft"], a["out"], a["ws"], a["wsb"], None)
+    assert partials(off=301) == 2          # shard past the vocabulary
+    assert partials(off=-1) == 2
+    assert partials(Vs=0) == 2
+    assert partials(K=32) == 2
+    assert partials(H=12) == 2             # rows not 16-byte pitched
+    assert partials(h=NULL) == 1
+    assert partials(out=NULL) == 1
+    assert partials(draft=NULL) == 1
+    assert partials(ws=NULL) == 1
+    assert partials(wsb=16) == 5
+    assert partials(w=0x2008) == 6         # weight not 16-byte aligned
+    assert partials(B=0) == 0              # empty batch: nothing to do
+
+
 def test_workspace_init_null(lib):
     assert lib.asd_workspace_init(None, 256, None) == 1
 
