@@ -38,15 +38,16 @@ CASES = [
 ]
 
 
+@pytest.mark.parametrize("resident", [False, True])
 @pytest.mark.parametrize("case", CASES)
-def test_blocks_equal_sequential_calls_and_oracle(asd, kernel, case):
+def test_blocks_equal_sequential_calls_and_oracle(asd, kernel, case, resident):
     nblk, B, K, V, dtype, budget, gate, cap = case
     logits, draft = _blocks(nblk, B, K, V, dtype, 31_000 + nblk * 100 + B)
     led_blk = asd.make_ledger(B, budget)
-    out = asd.verify_blocks(logits, draft, led_blk, gate, cap)
+    out = asd.verify_blocks(logits, draft, led_blk, gate, cap, resident=resident)
     led_seq = asd.make_ledger(B, budget)
     ws = asd.Workspace(B, K, V, asd.BF16 if dtype == torch.bfloat16 else asd.F32)
-    seq = [asd.verify(logits[i], draft[i], led_seq, gate, cap, workspace=ws) for i in range(nblk)]
+    seq = [asd.verify(logits[i], draft[i], led_seq, gate, cap, workspace=ws, resident=resident) for i in range(nblk)]
     torch.cuda.synchronize()
     for i in range(nblk):
         for key in ("accepted_len", "committed", "recovery", "row_argmax", "status"):

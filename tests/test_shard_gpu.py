@@ -24,7 +24,7 @@ def kernel(request, monkeypatch):
     return request.param
 
 
-def run_sharded(asd, logits, draft, bounds, ledger, gate, cap, misalign=0):
+def run_sharded(asd, logits, draft, bounds, ledger, gate, cap, misalign=0, resident=False):
     V = logits.shape[-1]
     parts = []
     for lo, hi in zip(bounds[:-1], bounds[1:]):
@@ -36,7 +36,7 @@ def run_sharded(asd, logits, draft, bounds, ledger, gate, cap, misalign=0):
             shard = buf
         else:
             shard = shard.contiguous()
-        parts.append(asd.shard_partials(shard, draft, lo, V))
+        parts.append(asd.shard_partials(shard, draft, lo, V, resident=resident))
     return asd.shard_combine(torch.stack(parts).contiguous(), draft, ledger, gate, cap, V)
 
 
@@ -59,7 +59,8 @@ def test_sharded_equals_unsharded_and_oracle(asd, kernel, case, misalign):
         draft[0, 1] = V + 3  # an out-of-range draft id
     led_s = asd.make_ledger(B, 4.0)
     led_u = asd.make_ledger(B, 4.0)
-    sh = run_sharded(asd, blk.logits, draft, bounds, led_s, 1.0, 2, misalign)
+    # the misaligned shards also pass ASD_RESIDENT_INPUTS (their copies were made before the calls)
+    sh = run_sharded(asd, blk.logits, draft, bounds, led_s, 1.0, 2, misalign, resident=bool(misalign))
     un = asd.verify(blk.logits, draft, led_u, 1.0, 2)
     torch.cuda.synchronize()
     for key in ("accepted_len", "committed", "recovery", "row_argmax", "status"):
