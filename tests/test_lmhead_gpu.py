@@ -247,3 +247,38 @@ def test_lmhead_sharded_partials_combine_to_the_unsharded_verify(asd, B, K, H, V
     for key in ("accepted_len", "committed", "recovery", "row_argmax", "status"):
         assert np.array_equal(sharded[key].cpu().numpy(), o[key]), f"oracle: {key}"
     assert np.array_equal(led_s.cpu().numpy().view(np.int32), o["ledger"].view(np.int32))
+
+
+def test_lmhead_verify_infinities_through_the_tensor_cores(asd):
+    """A +inf weight: where h is +1 the row's logit is +inf (it wins), where h is -1 it is -inf, and
+    0 x inf = NaN flags the request; every other output equals the fp64 oracle (IEEE on both sides)."""
+    B, K, H, V = 6, 4, 64, 700
+    inp = inputs.gen_lmhead_exact(B, K, H, V, 7500, "cuda")
+    K1 = K + 1
+    weight = inp.weight.clone()
+    weight[5, 0] = float("inf")
+    hidden = inp.hidden.clone()
+    sign = torch.tensor([1.0, 1.0, -1.0, -1.0, -1.0, 1.0], device="cuda").repeat_interleave(K1)
+    hidden[:, 0] = sign.to(torch.bfloat16)
+    hidden[4 * K1 + 2, 0] = 0.0            # request 4, row 2: 0 x inf = NaN
+    draft = inp.draft.clone()
+    draft[0, 0] = 5                        # matches an +inf argmax (its regret is inf - inf = NaN, unused)
+    ledger0 = np.array([[8.0, 0.0]] * B, np.float32)
+    led = torch.from_numpy(ledger0).cuda()
+    out = asd.lmhead_verify(hidden, weight, draft, led, 1.0, 2)
+    torch.cuda.synchronize()
+    T = B * K1
+    z64, z32 = oracle_logits(hidden, weight, range(T))
+    assert np.isposinf(z32[0, 5]) and np.isneginf(z32[2 * K1, 5]) and np.isnan(z32[4 * K1 + 2, 5])
+    o = oracle.verify(z32.reshape(B, K1, V), draft.cpu().numpy(), ledger0, 1.0, 2)
+    g = {k: v.cpu().numpy() for k, v in out.items()}
+    assert np.array_equal(g["status"], o["status"])
+    assert g["status"][4] & oracle.STATUS_NAN_LOGIT and g["accepted_len"][4] == 0
+    ok = g["status"] == 0
+    for key in ("accepted_len", "committed", "recovery", "row_argmax"):
+        assert np.array_equal(g[key][ok], o[key][ok]), key
+    assert np.all(g["row_argmax"][:2] == 5)
+    a, b = g["row_regret"][ok], o["row_regret"][ok]
+    assert np.array_equal(np.isnan(a), np.isnan(b))
+    assert np.array_equal(a[~np.isnan(a)].view(np.int32), b[~np.isnan(b)].view(np.int32))
+    assert np.array_equal(led.cpu().numpy().view(np.int32), o["ledger"].view(np.int32))
