@@ -435,3 +435,21 @@ def test_back_to_back_calls_carry_the_ledger(asd, shape, resident):
         ledger.copy_(torch.from_numpy(led0).cuda())
         graph.replay()
         check("graph")
+
+
+@pytest.mark.parametrize("cfg_id,dtype", [(1, torch.bfloat16), (3, torch.float32), (3, torch.bfloat16)])
+def test_zero_budget_is_strict_on_the_large_configs(asd, cfg_id, dtype):
+    """Budget 0 (Alg. 1's dispatch) equals asd_verify_strict and the oracle's strict mode bit for bit,
+    and leaves the ledger untouched, on the Qwen3-14B and the large-batch 129k workloads."""
+    cfg = inputs.CONFIGS[cfg_id]
+    B, K, V = cfg["B"], cfg["K"], cfg["V"]
+    for blk in range(2):
+        b = inputs.gen_block(B, K, V, dtype, inputs.seed_for(cfg_id, 40, blk), "cuda")
+        led = asd.make_ledger(B, 0.0, 0.0)
+        g = gpu_verify(asd, b.logits, b.draft, led, 1.0, 2)
+        s = gpu_verify(asd, b.logits, b.draft, None, 0, 0, strict=True)
+        o = oracle.verify(b.logits.cpu(), b.draft.cpu().numpy(), None, strict=True)
+        for key in ("accepted_len", "committed", "recovery", "row_argmax", "status"):
+            assert np.array_equal(g[key], s[key]), f"strict entry: {key}"
+            assert np.array_equal(g[key], o[key]), f"oracle strict: {key}"
+        assert np.array_equal(g["ledger"], np.zeros((B, 2), np.float32))
