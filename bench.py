@@ -39,6 +39,13 @@ B, K, V = 32, 8, 151936
 GATE, CAP, BUDGET = 1.0, 2, 8.0
 WORKLOAD = "qwen3-14b-verify: B=32 requests, K=8 draft tokens (288 target rows), V=151936, bf16 logits, " \
            "gate=1.0, cap=2, budget=8.0 carried across steps"
+
+
+def bench_config(world: int) -> dict:
+    """The workload, as both arms report it (the same dict, so the two lines compare like for like)."""
+    return {"workload": WORKLOAD, "B": B, "K": K, "V": V, "gate": GATE, "cap": CAP, "budget": BUDGET,
+            "parallelism": f"dp{world} (independent requests per rank)",
+            "l2": "inputs larger than L2: steps rotate over logit buffers totalling more than 4x the L2 size"}
 CSRC = os.path.join(ROOT, "paper_2608_03447_gb300", "csrc")
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
 # the sources each profiled kernel is built from (a recorded traffic figure is
@@ -70,12 +77,15 @@ def source_digest(kernel: str) -> str:
     return h.hexdigest()
 
 
-def recorded_traffic(kernel: str) -> float | None:
-    """DRAM bytes per launch from the committed ncu summary, if it is for the current kernel sources."""
+def recorded_traffic(kernel: str, workload: str | None = None) -> float | None:
+    """DRAM bytes per launch from the committed ncu summary (the headline workload's, or the named
+    workload's entry), if it is for the current kernel sources."""
     try:
         with open(TRAFFIC_FILE) as f:
             rec = json.load(f)[kernel]
-    except (OSError, ValueError, KeyError):
+        if workload is not None:
+            rec = rec["workloads"][workload]
+    except (OSError, ValueError, KeyError, TypeError):
         return None
     if rec.get("sources_sha256") != source_digest(kernel):
         return None
@@ -93,28 +103,43 @@ def bf16_peaks() -> dict:
         return {"burst": 1900.0, "sustained": 1700.0, "source": "fallback"}
 
 
-def run_lmhead(dev, iters: int = 20) -> dict:
-    """The fused LM-head + verify timed alone (burst peak): CUDA events around `iters` launches."""
+def run_lmhead(dev, clocks=None, iters: int = 20, sustain_s: float = 1.2) -> dict:
+    """The fused LM-head + verify timed alone: CUDA events around `iters` launches (burst peak), then a
+    sustained loop of about `sustain_s` seconds with the SM clock sampled, so that each time can be read
+    with the clock it ran at (time x median SM GHz separates a tiling change from clock drift)."""
     from paper_2608_03447_gb300 import asd, inputs
     inp = inputs.gen_lmhead(LM_B, LM_K, LM_H, LM_V, inputs.seed_for(4), dev)
     led = asd.make_ledger(LM_B, 8.0, 0.0, dev)
     ws = asd.lmhead_workspace(LM_B, LM_K, LM_V, LM_H, dev)
     out = asd.alloc_outputs(LM_B, LM_K, dev)
     out["row_top"] = torch.empty(LM_B, LM_K + 1, device=dev)
-    for _ in range(3):
-        asd.lmhead_verify(inp.hidden, inp.weight, inp.draft, led, 1.0, 2, workspace=ws, out=out)
-    torch.cuda.synchronize(dev)
     stream = torch.cuda.current_stream(dev)
-    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    start.record(stream)
-    for _ in range(iters):
+
+    def launch():
         asd.lmhead_verify(inp.hidden, inp.weight, inp.draft, led, 1.0, 2, workspace=ws, out=out)
-    end.record(stream)
-    end.synchronize()
-    ms = start.elapsed_time(end) / iters
+
+    def timed(n):
+        start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t0 = time.time()
+        start.record(stream)
+        for _ in range(n):
+            launch()
+        end.record(stream)
+        end.synchronize()
+        return start.elapsed_time(end) / n, t0, time.time()
+
+    for _ in range(3):
+        launch()
+    torch.cuda.synchronize(dev)
+    ms, tb0, tb1 = timed(iters)
+    n_sus = max(iters, int(sustain_s / (ms * 1e-3)))
+    ms_sus, ts0, ts1 = timed(n_sus)
     flop = 2.0 * LM_B * (LM_K + 1) * LM_H * LM_V
     tflops = flop / (ms * 1e-3) / 1e12
+    tflops_sus = flop / (ms_sus * 1e-3) / 1e12
     pk = bf16_peaks()
+    clk_b = clocks.window(tb0, tb1) if clocks is not None else {"sm_mhz": None}
+    clk_s = clocks.window(ts0, ts1) if clocks is not None else {"sm_mhz": None}
     # one of four tensor-parallel ranks: its quarter of W, the partials (the all-gather and the
     # combine follow; the combine is timed with the sharded verify row)
     S = 4
@@ -134,21 +159,31 @@ def run_lmhead(dev, iters: int = 20) -> dict:
     ms_rank = s2.elapsed_time(e2) / iters
     del shard
     rank_tflops = flop / S / (ms_rank * 1e-3) / 1e12
-    return {"workload": LM_WORKLOAD, "ms_per_step": ms, "rows_per_s": LM_B * (LM_K + 1) / (ms * 1e-3),
-            "launches": iters,
-            "per_rank_of_4": {"ms": ms_rank, "tflops": rank_tflops, "frac": rank_tflops / pk["burst"],
-                              "workload": f"asd_lmhead_partials on a {vs} x {LM_H} shard of W (one of {S} "
-                                          "tensor-parallel ranks), 576 rows"},
-            "roofline": {"bound": "tensor", "achieved": tflops, "peak": pk["burst"], "unit": "TFLOP/s",
-                         "frac": tflops / pk["burst"], "peak_kind": "burst (kernel timed alone)",
-                         "peak_source": pk["source"], "traffic": recorded_traffic("lmhead_verify_kernel"),
-                         "kernel": "lmhead_verify_kernel", "algorithmic_flop_per_launch": flop}}
+
+    def ghz_ms(t, c):
+        return None if c.get("sm_mhz") is None else t * c["sm_mhz"] / 1e3
+
+    summary = {"bound": "tensor", "achieved": tflops, "peak": pk["burst"], "unit": "TFLOP/s",
+               "frac": tflops / pk["burst"], "ms": ms, "sm_mhz": clk_b.get("sm_mhz"),
+               "ms_x_ghz": ghz_ms(ms, clk_b),
+               "sustained": {"ms": ms_sus, "achieved": tflops_sus, "peak": pk["sustained"],
+                             "frac": tflops_sus / pk["sustained"], "sm_mhz": clk_s.get("sm_mhz"),
+                             "ms_x_ghz": ghz_ms(ms_sus, clk_s), "launches": n_sus,
+                             "reasons": clk_s.get("reasons")},
+               "traffic": recorded_traffic("lmhead_verify_kernel"), "kernel": "lmhead_verify_kernel",
+               "algorithmic_flop_per_launch": flop, "peak_source": pk["source"]}
+    detail = {"workload": LM_WORKLOAD, "ms_per_step": ms, "rows_per_s": LM_B * (LM_K + 1) / (ms * 1e-3),
+              "launches": iters,
+              "per_rank_of_4": {"ms": ms_rank, "tflops": rank_tflops, "frac": rank_tflops / pk["burst"],
+                                "workload": f"asd_lmhead_partials on a {vs} x {LM_H} shard of W (one of {S} "
+                                            "tensor-parallel ranks), 576 rows"}}
+    return {"summary": summary, "detail": detail}
 
 
 class ClockSampler:
     """nvidia-smi clock / throttle sampling in the background (200 ms period)."""
 
-    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+    QUERY = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
@@ -173,32 +208,46 @@ class ClockSampler:
     def mark_end(self):
         self.t1 = time.time()
 
-    def stop(self) -> dict:
+    def _rows(self):
+        """(unix time, sm MHz, max MHz, reason names) per sample."""
+        self.file.flush()
+        self.file.seek(0)
+        out = []
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.file.read().strip().splitlines():
+            r = [x.strip() for x in line.split(",")]
+            try:
+                t = time.mktime(time.strptime(r[0].split(".")[0], "%Y/%m/%d %H:%M:%S"))
+                t += float("0." + r[0].split(".")[1]) if "." in r[0] else 0.0
+                out.append((t, float(r[1]), float(r[2]),
+                            {n for n, v in zip(names, r[5:9]) if v.lower() in ("active", "1")}))
+            except (ValueError, IndexError):
+                continue
+        return out
+
+    def window(self, t0: float, t1: float, min_samples: int = 1) -> dict:
+        """Median SM clock and throttle reasons of the samples taken in [t0, t1]."""
+        rows = [r for r in self._rows() if t0 - 0.25 <= r[0] <= t1 + 0.25]
+        if len(rows) < min_samples:
+            return {"sm_mhz": None, "samples": len(rows)}
+        return {"sm_mhz": statistics.median(r[1] for r in rows), "sm_max_mhz": max(r[2] for r in rows),
+                "reasons": sorted(set().union(*(r[3] for r in rows))), "samples": len(rows)}
+
+    def stop(self) -> None:
         if self.proc is None:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+            return
         time.sleep(0.25)
         self.proc.terminate()
         try:
             self.proc.wait(timeout=5)
         except subprocess.TimeoutExpired:
             self.proc.kill()
-        self.file.flush()
-        self.file.seek(0)
-        rows = [r.split(",") for r in self.file.read().strip().splitlines() if r.strip()]
-        os.unlink(self.file.name)
-        sm, smax, reasons = [], [], set()
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for r in rows:
-            try:
-                sm.append(float(r[1]))
-                smax.append(float(r[2]))
-            except (ValueError, IndexError):
-                continue
-            for name, val in zip(names, r[5:9]):
-                if val.strip().lower() in ("active", "1"):
-                    reasons.add(name)
-        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
-                "reasons": sorted(reasons), "samples": len(sm)}
+
+    def close(self) -> None:
+        try:
+            os.unlink(self.file.name)
+        except OSError:
+            pass
 
 
 def dist_env():
@@ -266,7 +315,7 @@ def run_reference(args) -> None:
         "impl": "reference", "metric": METRIC, "value": rows_per_s, "unit": "rows/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": WORKLOAD, "B": B, "K": K, "V": V, "l2": "host memory (CPU oracle)"},
+        "config": bench_config(world),
         "cpu_baseline": {"value": rows_per_s, "unit": "rows/s", "cores": cores, "kind": "oracle",
                          "sample": f"{args.steps} full blocks of {B}x{K + 1}x{V} bf16, one request per thread"},
         "e2e": {"value": rows_per_s, "unit": "rows/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -370,7 +419,6 @@ def run_gpu(args) -> None:
     end.synchronize()
     barrier()
     clocks.mark_end()
-    clk = clocks.stop()
     ms_max = max_over_ranks(start.elapsed_time(end), dev, world)
     sec_per_step = ms_max / 1e3 / steps
     rows_per_step = B * (K + 1)
@@ -396,62 +444,120 @@ def run_gpu(args) -> None:
     interleaved = {k: {"median_us": float(np.median(v)), "best_us": float(min(v))} for k, v in per.items()}
     del graph_strict
 
-    # the same steps without the flag: each row stage reads nothing before the previous kernel completes
-    # (what a call right behind a producer kernel of its logits gets)
+    # the lone call: the same steps without the flag, each row stage reading nothing before the previous
+    # kernel completes (what a call right behind a producer kernel of its logits gets); graphs of 512
     wl.resident = False
-    graph_dflt = wl.capture(G, first=0)
+    G_lone = 512
+    graph_lone = wl.capture(G_lone, first=0)
     wl.reset_ledger()
-    graph_dflt.replay()
+    graph_lone.replay()
     torch.cuda.synchronize(dev)
-    s_d, e_d = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    s_d.record(stream)
-    graph_dflt.replay()
-    e_d.record(stream)
-    e_d.synchronize()
-    default_us = s_d.elapsed_time(e_d) * 1e3 / G
-    del graph_dflt
+    lone = []
+    for _ in range(3):
+        s_d, e_d = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s_d.record(stream)
+        graph_lone.replay()
+        e_d.record(stream)
+        e_d.synchronize()
+        lone.append(s_d.elapsed_time(e_d) * 1e3 / G_lone)
+    lone_us = float(np.median(lone))
+    del graph_lone
     wl.resident = True
     wl.reset_ledger()
+
+    # the allocation-free entry point on the same steps, eager (it clears its scratch before each call)
+    noalloc = run_noalloc(wl, dev) if rank == 0 else None
 
     # end to end through the public API from pinned host buffers (copies inside the timed region)
     e2e = run_e2e(wl, dev, steps=max(10, min(steps, 200)), world=world)
 
-    lm = run_lmhead(dev) if rank == 0 else None
+    lm = run_lmhead(dev, clocks) if rank == 0 else None
     nxt = run_next_rows(wl, dev) if rank == 0 else None
     other = run_other_configs(dev) if rank == 0 and args.configs else None
+    clocks.stop()
+    timed = clocks.window(clocks.t0, clocks.t1)
+    if timed["sm_mhz"] is not None:
+        clk = dict(timed, window="timed region")
+    else:
+        clk = dict(clocks.window(t_soak, clocks.t1),
+                   window="1 s of the same step graph ending at the timed region (which is shorter than "
+                          "the 200 ms sampling period)")
+    clocks.close()
     if rank == 0:
         pk = peaks()
         cpu = cpu_baseline(wl) if world == 1 else None
+        lone_gbs = bytes_per_launch / (lone_us * 1e-6) / 1e9
+        roofline = {
+            "bound": "hbm", "achieved": achieved_gbs, "peak": pk["hbm_gbs"], "unit": "GB/s",
+            "frac": achieved_gbs / pk["hbm_gbs"], "traffic": recorded_traffic("verify_tma_kernel"),
+            "peak_source": pk["source"], "kernel": "verify_tma_kernel<bf16> + select_kernel, resident inputs",
+            "algorithmic_bytes_per_launch": bytes_per_launch, "pct_of_8tbs": achieved_gbs / NOMINAL_HBM_GBS,
+            "launch": f"CUDA graphs of {G} steps, {asd.verify_launches(B, K, V, asd.BF16)} kernels per step; "
+                      "ASD_RESIDENT_INPUTS (buffers written before the timed region; consecutive steps overlap)",
+            "lone_call": {"us_per_step": lone_us, "achieved": lone_gbs, "frac": lone_gbs / pk["hbm_gbs"],
+                          "launch": f"graphs of {G_lone} steps without ASD_RESIDENT_INPUTS: each step waits "
+                                    "for the previous kernel before its first read"},
+        }
+        if lm is not None:
+            roofline["fused_lmhead"] = lm["summary"]
+        if other is not None:
+            roofline["other_configs"] = {k: {"us": round(v["us_per_step"], 2),
+                                             "frac": round(v["roofline"]["frac"], 3),
+                                             "traffic": v["roofline"]["traffic"]}
+                                         for k, v in other.items() if "roofline" in v}
         line = {
             "metric": METRIC, "value": value, "unit": "rows/s", "n_gpus": world, "steps": steps,
             "warmup": warmup, "ms_per_step": sec_per_step * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": WORKLOAD, "B": B, "K": K, "V": V, "gate": GATE, "cap": CAP,
-                       "budget": BUDGET, "parallelism": f"dp{world} (independent requests per rank)",
-                       "l2": f"inputs rotate over {wl.nbuf} logit buffers = "
-                             f"{wl.nbuf * bytes_per_launch / 1e6:.0f} MB (> 4x the {l2_bytes(dev) / 1e6:.0f} MB L2)",
-                       "launch": f"CUDA graphs of {G} steps, "
-                                 f"{asd.verify_launches(B, K, V, asd.BF16)} kernels per step",
-                       "inputs": "ASD_RESIDENT_INPUTS (buffers written before the timed region; consecutive "
-                                 "steps overlap)"},
-            "without_resident_flag_us_per_step": default_us,
-            "interleaved_graphs_us_per_step": interleaved,
-            "hbm_gbs": achieved_gbs, "pct_of_8tbs": achieved_gbs / NOMINAL_HBM_GBS,
-            "roofline": {"bound": "hbm", "achieved": achieved_gbs, "peak": pk["hbm_gbs"], "unit": "GB/s",
-                         "frac": achieved_gbs / pk["hbm_gbs"], "traffic": recorded_traffic("verify_tma_kernel"),
-                         "peak_source": pk["source"], "kernel": "verify_tma_kernel<bf16, asd>",
-                         "algorithmic_bytes_per_launch": bytes_per_launch},
+            "config": bench_config(world),
+            "roofline": roofline,
             "clocks": clk,
             "e2e": e2e,
             "gpu_launches": steps * asd.verify_launches(B, K, V, asd.BF16),
             "cpu_baseline": cpu,
-            "fused_lmhead": lm,
+            "interleaved_graphs_us_per_step": interleaved,
+            "noalloc": noalloc,
+            "fused_lmhead": lm["detail"] if lm is not None else None,
             "next_rows": nxt,
             "other_configs": other,
         }
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
+
+
+def run_noalloc(wl, dev, calls: int = 200) -> dict:
+    """asd_verify_noalloc against asd_verify on the same steps, both eager on one stream."""
+    from paper_2608_03447_gb300 import asd
+    stream = torch.cuda.current_stream(dev)
+    out = asd.alloc_outputs(B, K, dev)
+
+    def run(fn):
+        for i in range(3):
+            fn(i)
+        torch.cuda.synchronize(dev)
+        s_, e_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s_.record(stream)
+        for i in range(calls):
+            fn(i)
+        e_.record(stream)
+        e_.synchronize()
+        return s_.elapsed_time(e_) * 1e3 / calls
+
+    def with_ws(i):
+        k = i % wl.nbuf
+        asd.verify(wl.logits[k], wl.drafts[k], wl.ledger, GATE, CAP, wl.workspace, out, resident=True)
+
+    def without(i):
+        k = i % wl.nbuf
+        asd.verify_noalloc(wl.logits[k], wl.drafts[k], wl.ledger, GATE, CAP, out, resident=True)
+
+    us_ws = run(with_ws)
+    us_na = run(without)
+    wl.reset_ledger()
+    return {"verify_us_per_call": us_ws, "noalloc_us_per_call": us_na,
+            "note": f"{calls} eager calls each (host launch overhead included), resident inputs; the "
+                    "allocation-free call clears its scratch with a memset before its kernels"}
 
 
 def run_e2e(wl, dev, steps: int, world: int) -> dict:
@@ -530,14 +636,16 @@ def run_other_configs(dev) -> dict:
     from paper_2608_03447_gb300.workload import VerifyWorkload
     pk = peaks()
     cases = [
-        ("tiny-fp32", 0, 4, 8, 1024, torch.float32, 1.0, 2, 4.0, inputs.MIX_DEFAULT),
+        ("tiny-fp32", 0, 4, 8, 1024, torch.float32, 1.0, 2, 4.0, inputs.MIX_DEFAULT, None),
         ("budget-cap-sweep bf16 (g=1, M=2, budget=8)", 2, 128, 16, 151936, torch.bfloat16, 1.0, 2, 8.0,
-         inputs.MIX_DEFAULT),
-        ("large-batch-129k fp32 (p_hit=0.7)", 3, 256, 4, 129280, torch.float32, 1.0, 1, 4.0, inputs.mix_for_hit(0.7)),
-        ("large-batch-129k bf16 (p_hit=0.7)", 3, 256, 4, 129280, torch.bfloat16, 1.0, 1, 4.0, inputs.mix_for_hit(0.7)),
+         inputs.MIX_DEFAULT, "budget-cap-sweep"),
+        ("large-batch-129k fp32 (p_hit=0.7)", 3, 256, 4, 129280, torch.float32, 1.0, 1, 4.0, inputs.mix_for_hit(0.7),
+         "large-batch-129k-f32"),
+        ("large-batch-129k bf16 (p_hit=0.7)", 3, 256, 4, 129280, torch.bfloat16, 1.0, 1, 4.0, inputs.mix_for_hit(0.7),
+         "large-batch-129k-bf16"),
     ]
     out = {}
-    for name, cfg, b, k, v, dtype, gate, cap, budget, mix in cases:
+    for name, cfg, b, k, v, dtype, gate, cap, budget, mix, traffic_key in cases:
         wl = VerifyWorkload(b, k, v, dtype, gate, cap, budget, config=cfg, mix=mix, device=dev, resident=True)
         steps = 200 if wl.bytes_per_step > (1 << 26) else 2000
         graph = wl.capture(steps)
@@ -558,7 +666,9 @@ def run_other_configs(dev) -> dict:
                "kernels_per_step": asd.verify_launches(b, k, v, code), "buffers": wl.nbuf, "steps": steps}
         if wl.bytes_per_step > (1 << 26):
             rec["roofline"] = {"bound": "hbm", "achieved": gbs, "peak": pk["hbm_gbs"], "unit": "GB/s",
-                               "frac": gbs / pk["hbm_gbs"]}
+                               "frac": gbs / pk["hbm_gbs"],
+                               "traffic": recorded_traffic("verify_tma_kernel", traffic_key),
+                               "algorithmic_bytes_per_launch": wl.bytes_per_step}
         else:
             rec["bound"] = "launch latency (147 KB per call)"
         out[name] = rec
@@ -669,18 +779,68 @@ def run_next_rows(wl, dev) -> dict:
     return out
 
 
+CASES = {
+    # name: (config, B, K, V, dtype, resident, forced path)
+    "verify-qwen3": (1, 32, 8, 151936, "bf16", True, "auto"),
+    "verify-qwen3-lone": (1, 32, 8, 151936, "bf16", False, "auto"),
+    "verify-qwen3-stream": (1, 32, 8, 151936, "bf16", True, "stream"),
+    "verify-sweep": (2, 128, 16, 151936, "bf16", True, "auto"),
+    "verify-129k-f32": (3, 256, 4, 129280, "f32", True, "auto"),
+    "verify-129k-bf16": (3, 256, 4, 129280, "bf16", True, "auto"),
+    "verify-tiny": (0, 4, 8, 1024, "f32", True, "auto"),
+}
+
+
+def run_case(name: str, launches: int) -> None:
+    """A few launches of one workload and nothing else, for a profiler to capture (one GPU, small)."""
+    from paper_2608_03447_gb300 import asd, inputs
+    from paper_2608_03447_gb300.workload import VerifyWorkload
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    asd.load()
+    if name == "lmhead":
+        inp = inputs.gen_lmhead(LM_B, LM_K, LM_H, LM_V, inputs.seed_for(4), dev)
+        led = asd.make_ledger(LM_B, 8.0, 0.0, dev)
+        for _ in range(2 + launches):
+            asd.lmhead_verify(inp.hidden, inp.weight, inp.draft, led, 1.0, 2)
+        torch.cuda.synchronize(dev)
+        print(json.dumps({"case": name, "launches": 2 + launches}))
+        return
+    control = name.startswith("torch-amax:")
+    cfg, b, k, v, dt, resident, path = CASES[name.split(":", 1)[1] if control else name]
+    dtype = torch.bfloat16 if dt == "bf16" else torch.float32
+    mix = inputs.mix_for_hit(0.7) if cfg == 3 else inputs.MIX_DEFAULT
+    wl = VerifyWorkload(b, k, v, dtype, GATE, CAP, BUDGET, config=cfg, mix=mix, device=dev, resident=resident)
+    asd.set_launch_options(path=path)
+    for i in range(2 + launches):
+        if control:  # the same bytes through a library row reduction, for comparison
+            torch.amax(wl.logits[i % wl.nbuf], dim=-1)
+        else:
+            wl.step(i)
+    torch.cuda.synchronize(dev)
+    asd.reset_launch_options()
+    print(json.dumps({"case": name, "launches": 2 + launches, "bytes_per_launch": wl.bytes_per_step,
+                      "buffers": wl.nbuf}))
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="asd", choices=["asd", "reference"])
+    ap.add_argument("--case", default=None,
+                    help="run only a few launches of one workload (for ncu): " + ", ".join(
+                        list(CASES) + ["lmhead"] + [f"torch-amax:{c}" for c in CASES]))
+    ap.add_argument("--launches", type=int, default=3)
     ap.add_argument("--no-configs", dest="configs", action="store_false",
                     help="skip timing the other workloads (configs 0, 2, 3)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
-    if args.impl == "reference":
+    if args.case is not None:
+        run_case(args.case, args.launches)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_gpu(args)

@@ -92,6 +92,10 @@ enum {
 #define ASD_STATUS_NAN_LOGIT 2u   /* a NaN among the request's K+1 logit rows */
 #define ASD_STATUS_BAD_LEDGER 4u  /* budget < 0 or NaN, spent < 0 or NaN, spent > budget */
 #define ASD_STATUS_OVERFLOW 8u    /* asd_commit: the token history has no room for the block */
+#define ASD_STATUS_INCOMPLETE 16u /* the workspace's error word was set when the request was
+                                   * selected (asd_workspace_error): a kernel gave up waiting on
+                                   * its copy pipeline, so row results may be missing. Set for
+                                   * every request of such a call until asd_workspace_init. */
 
 /* Largest draft length: one warp lane per target row of a block. */
 #define ASD_MAX_K 31
@@ -225,13 +229,19 @@ int asd_lmhead_logits(const void* hidden, const void* weight, int H, int T, int 
  * ASD_ERR_SCRATCH_LIMIT and launches nothing.
  * Set-up: the first call made with a given device current looks up the
  * array's device address (cudaGetSymbolAddress); make that first call outside
- * any stream capture.
+ * any stream capture. The address is kept for the life of the process:
+ * cudaDeviceReset unloads the library's device code, so after it this entry
+ * point must not be called again in that process.
  * Each call clears the part of the array it uses (cudaMemsetAsync on
- * `stream`) and then launches the verify kernel. Every call on every stream
- * shares the one array: calls that can overlap on the GPU (different streams,
- * no ordering between them) race and give wrong results. Order them on one
- * stream. Allocates nothing: no cudaMalloc, cudaFree or allocating library
- * call.
+ * `stream`, which also clears the array's error word) and then launches the
+ * verify kernels. Every call on every stream shares the one array: calls that
+ * can overlap on the GPU (different streams, no ordering between them) race
+ * and give wrong results. Order them on one stream. Allocates nothing: no
+ * cudaMalloc, cudaFree or allocating library call.
+ * Failure report: the array's error word is not readable by the caller, so a
+ * call whose kernels gave up waiting on their copy pipeline (the bounded wait
+ * of asd_workspace_error) flags every request ASD_STATUS_INCOMPLETE in
+ * status[b] instead (a = 0, ledger kept); pass a status array to see it.
  */
 int asd_verify_noalloc(const void* logits, int dtype, int B, int K, int V, const int32_t* draft,
                        asd_ledger* ledger, float gate, int cap, int32_t* accepted_len,
@@ -345,6 +355,33 @@ int asd_host_alias(const void* host, void** device);
  * shape (1 or 2: the row stage, and for large inputs a separate selection
  * kernel launched right behind it); 0 for B = 0. For accounting only. */
 int asd_verify_launches(int B, int K, int V, int dtype, int* launches);
+
+/* Launch options of the logit-streaming entry points (asd_verify,
+ * asd_verify_strict, asd_verify_blocks, asd_shard_partials, asd_verify_noalloc).
+ * The paper has no counterpart: these choose among kernels that compute the
+ * same results bit for bit, for tests that cover each kernel and for
+ * measurements; the defaults (all fields 0) are what production calls want.
+ *   path          ASD_PATH_AUTO picks the row-stage kernel by input size (the
+ *                 one-CTA-per-request kernel below 1 MB when a request fits
+ *                 it, the register-streaming kernel for other small inputs,
+ *                 the TMA pipeline from 1 MB); the others force one (a forced
+ *                 ASD_PATH_SMALL falls back to AUTO where the shape does not
+ *                 fit it).
+ *   fused_select  1: the TMA row stage runs the selection itself (the CTA that
+ *                 completes a request selects it) instead of launching
+ *                 select_kernel right behind it.
+ *   no_pdl        1: launch without programmatic dependent launch.
+ * Process-wide; each call reads the options once when it is issued, and a CUDA
+ * graph keeps the kernels chosen at capture. asd_set_launch_options(NULL)
+ * restores the defaults. Returns ASD_ERR_CONTROL for an unknown path. */
+enum { ASD_PATH_AUTO = 0, ASD_PATH_SMALL = 1, ASD_PATH_STREAM = 2, ASD_PATH_TMA = 3 };
+typedef struct {
+  int path;
+  int fused_select;
+  int no_pdl;
+} asd_launch_options;
+int asd_set_launch_options(const asd_launch_options* options);
+int asd_get_launch_options(asd_launch_options* options);
 
 /* Human-readable text of a return code. Never NULL. */
 const char* asd_status_string(int code);

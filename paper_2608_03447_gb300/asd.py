@@ -31,6 +31,7 @@ STATUS_DRAFT_RANGE = 1
 STATUS_NAN_LOGIT = 2
 STATUS_BAD_LEDGER = 4
 STATUS_OVERFLOW = 8
+STATUS_INCOMPLETE = 16
 MAX_K = 31
 RESIDENT_INPUTS = 0x100  # ASD_RESIDENT_INPUTS, ORed into the dtype code
 INT32_MAX = 2**31 - 1
@@ -90,7 +91,35 @@ def _declare(lib: ctypes.CDLL) -> ctypes.CDLL:
     lib.asd_lmhead_logits.restype = i32
     lib.asd_lmhead_partials.argtypes = [vp, vp, i32, i32, i32, i32, i32, i32, vp, vp, vp, sz, vp]
     lib.asd_lmhead_partials.restype = i32
+    lib.asd_set_launch_options.argtypes = [vp]
+    lib.asd_set_launch_options.restype = i32
+    lib.asd_get_launch_options.argtypes = [vp]
+    lib.asd_get_launch_options.restype = i32
     return lib
+
+
+class _LaunchOptions(ctypes.Structure):
+    _fields_ = [("path", ctypes.c_int), ("fused_select", ctypes.c_int), ("no_pdl", ctypes.c_int)]
+
+
+PATHS = {"auto": 0, "small": 1, "stream": 2, "tma": 3}
+
+
+def set_launch_options(path: str = "auto", fused_select: bool = False, pdl: bool = True) -> None:
+    """asd_set_launch_options: which row-stage kernel the verify calls use (process-wide)."""
+    opt = _LaunchOptions(PATHS[path], int(fused_select), int(not pdl))
+    _check("asd_set_launch_options", load().asd_set_launch_options(ctypes.byref(opt)))
+
+
+def get_launch_options() -> dict:
+    opt = _LaunchOptions()
+    _check("asd_get_launch_options", load().asd_get_launch_options(ctypes.byref(opt)))
+    names = {v: k for k, v in PATHS.items()}
+    return {"path": names[opt.path], "fused_select": bool(opt.fused_select), "pdl": not opt.no_pdl}
+
+
+def reset_launch_options() -> None:
+    _check("asd_set_launch_options", load().asd_set_launch_options(None))
 
 
 def load(path: str = LIBRARY) -> ctypes.CDLL:

@@ -230,11 +230,21 @@ __device__ __forceinline__ void select_block(const VerifyParams& p, long long vb
 // from block to block, and written once. Runs in one warp.
 // Vocabulary-shard mode: instead of selecting, hand each row's reduction of
 // this shard to the combine step (global index, exact top, draft logit).
+// ASD_STATUS_INCOMPLETE when the workspace's error word is set: a kernel that
+// used this workspace gave up waiting on its copy pipeline, so row results may
+// be missing (every lane gets the same answer).
+__device__ __forceinline__ unsigned workspace_failed(const VerifyParams& p, int lane) {
+  unsigned err = 0;
+  if (lane == 0 && p.error) err = __ldcg(p.error);
+  return __shfl_sync(kFull, err, 0) ? ASD_STATUS_INCOMPLETE : 0u;
+}
+
 template <typename T>
 __device__ void emit_partials(const VerifyParams& p, int b, int lane) {
   const int K = p.K, K1 = p.K + 1;
   const T* z = static_cast<const T*>(p.logits);
   BlockInputs in = load_block(p, b, lane);
+  in.flags |= workspace_failed(p, lane);
   if (lane < K1) {
     const long long row = static_cast<long long>(b) * K1 + lane;
     const uint32_t local = 0xffffffffu - static_cast<uint32_t>(in.key);
@@ -267,12 +277,14 @@ __device__ void select_request(const VerifyParams& p, int b, int lane) {
   }
   budget = __shfl_sync(kFull, budget, 0);
   spent = __shfl_sync(kFull, spent, 0);
+  const unsigned incomplete = workspace_failed(p, lane);
   bool wrote = false;
   BlockInputs cur = load_block(p, b, lane);
   for (int i = 0; i < p.nblk; ++i) {
     const long long vb = static_cast<long long>(i) * p.B + b;
     BlockInputs next = cur;
     if (i + 1 < p.nblk) next = load_block(p, vb + p.B, lane);  // in flight while this block is selected
+    cur.flags |= incomplete;
     select_block<T, kStrict>(p, vb, cur, budget, spent, wrote, lane);
     cur = next;
   }

@@ -25,7 +25,6 @@
 
 #include <cstdlib>
 #include <atomic>
-#include <cstring>
 #include <mutex>
 
 #include "asd.h"
@@ -324,7 +323,7 @@ __global__ void __launch_bounds__(kSmallThreads) verify_small_kernel(const __gri
   in.key = lane < K1 ? s_key[lane] : 0ull;
   in.x = lane < K ? __ldg(p.draft + static_cast<long long>(b) * K + lane) : -1;
   in.zx = lane < K ? s_zx[lane] : 0.0f;
-  in.flags = s_flags;
+  in.flags = s_flags | workspace_failed(p, lane);
   in.top = ordered_value(static_cast<uint32_t>(in.key >> 32));
   in.top_exact = false;
   budget = __shfl_sync(kFull, budget, 0);
@@ -874,12 +873,24 @@ struct DeviceInfo {
   std::atomic<bool> tma_ready[8] = {};
 };
 
-// The TMA path's selection runs in its own kernel right behind the row stage
-// (see select_kernel); ASD_VERIFY_SPLIT=0 in the environment keeps it inside
-// the row-stage kernel instead (last-CTA-done), for comparison and testing.
-bool use_split() {
-  const char* env = getenv("ASD_VERIFY_SPLIT");
-  return !(env && env[0] == '0');
+// Launch options (asd_set_launch_options): process-wide, read once per call,
+// so a call (and a CUDA graph captured from it) sees one consistent set.
+std::atomic<int> g_path{ASD_PATH_AUTO};
+std::atomic<int> g_flags{0};  // bit 0: selection inside the row stage, bit 1: no PDL
+
+struct LaunchOptions {
+  int path;
+  bool split;  // the TMA path's selection runs in select_kernel, right behind the row stage
+  bool pdl;    // launches carry the programmatic-serialization attribute
+};
+
+LaunchOptions launch_options() {
+  const int f = g_flags.load(std::memory_order_relaxed);
+  LaunchOptions o;
+  o.path = g_path.load(std::memory_order_relaxed);
+  o.split = (f & 1) == 0;
+  o.pdl = (f & 2) == 0;
+  return o;
 }
 
 // SM count of the current device, and the one-time dynamic shared memory
@@ -903,7 +914,7 @@ int device_info(int* dev_out, DeviceInfo** info_out) {
 }
 
 template <typename T, bool kStrict>
-int launch_tma(VerifyParams& p, cudaStream_t stream) {
+int launch_tma(VerifyParams& p, const LaunchOptions& opt, cudaStream_t stream) {
   constexpr int VN = Elem<T>::kVec;
   constexpr long long kMinPerCta = 2LL * kTmaChunkBytes / static_cast<long long>(sizeof(T));
   const uintptr_t addr = reinterpret_cast<uintptr_t>(p.logits);
@@ -915,7 +926,7 @@ int launch_tma(VerifyParams& p, cudaStream_t stream) {
   DeviceInfo* info = nullptr;
   int rc = device_info(&dev, &info);
   if (rc != ASD_OK) return rc;
-  const bool split = use_split();
+  const bool split = opt.split;
   const int slot = (sizeof(T) == 2 ? 2 : 0) + (kStrict ? 1 : 0) + (split ? 4 : 0);
   if (!info->tma_ready[slot].load(std::memory_order_acquire)) {
     auto kernel = split ? verify_tma_kernel<T, kStrict, true> : verify_tma_kernel<T, kStrict, false>;
@@ -947,8 +958,7 @@ int launch_tma(VerifyParams& p, cudaStream_t stream) {
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
-  const char* env = getenv("ASD_VERIFY_PDL");
-  if (!(env && env[0] == '0')) {
+  if (opt.pdl) {
     cfg.attrs = attr;
     cfg.numAttrs = 1;
   }
@@ -973,19 +983,18 @@ int launch_tma(VerifyParams& p, cudaStream_t stream) {
 // kTmaMinBytes; below that, one CTA per request when a request fits one round
 // of loads of a CTA (single blocks, no vocabulary shard), else the
 // register-streaming kernel (fewer, shorter warps start faster on small
-// inputs). ASD_VERIFY_KERNEL=stream|tma|small in the environment overrides the
-// choice (the tests use it to cover every kernel); `small` falls back to the
-// default when the shape does not qualify.
+// inputs). The launch options can force a kernel (the tests use that to cover
+// every kernel); a forced `small` falls back to the default when the shape does
+// not qualify.
 constexpr long long kTmaMinBytes = 1LL << 20;
 
 enum class Path { kSmall, kStream, kTma };
 
-Path choose_path(long long bytes, long long request_bytes, int K, bool single_block) {
+Path choose_path(int forced, long long bytes, long long request_bytes, int K, bool single_block) {
   const bool small_ok = single_block && K + 1 <= 32 && request_bytes <= kSmallMaxRequestBytes;
-  const char* env = getenv("ASD_VERIFY_KERNEL");
-  if (env && strcmp(env, "tma") == 0) return Path::kTma;
-  if (env && strcmp(env, "stream") == 0) return Path::kStream;
-  if (env && strcmp(env, "small") == 0 && small_ok) return Path::kSmall;
+  if (forced == ASD_PATH_TMA) return Path::kTma;
+  if (forced == ASD_PATH_STREAM) return Path::kStream;
+  if (forced == ASD_PATH_SMALL && small_ok) return Path::kSmall;
   if (bytes >= kTmaMinBytes) return Path::kTma;
   return small_ok ? Path::kSmall : Path::kStream;
 }
@@ -993,9 +1002,10 @@ Path choose_path(long long bytes, long long request_bytes, int K, bool single_bl
 template <typename T, bool kStrict>
 int launch(VerifyParams& p, cudaStream_t stream) {
   const long long request_bytes = static_cast<long long>(p.K + 1) * p.V * static_cast<long long>(sizeof(T));
-  const Path path = choose_path(p.total * static_cast<long long>(sizeof(T)), request_bytes, p.K,
+  const LaunchOptions opt = launch_options();
+  const Path path = choose_path(opt.path, p.total * static_cast<long long>(sizeof(T)), request_bytes, p.K,
                                 p.nblk == 1 && !p.partials);
-  if (path == Path::kTma) return launch_tma<T, kStrict>(p, stream);
+  if (path == Path::kTma) return launch_tma<T, kStrict>(p, opt, stream);
   constexpr int VN = Elem<T>::kVec;
   const uintptr_t addr = reinterpret_cast<uintptr_t>(p.logits);
   if (addr % sizeof(T) != 0) return ASD_ERR_ALIGN;
@@ -1011,8 +1021,7 @@ int launch(VerifyParams& p, cudaStream_t stream) {
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
-    const char* env = getenv("ASD_VERIFY_PDL");
-    if (!(env && env[0] == '0')) {
+    if (opt.pdl) {
       cfg.attrs = attr;
       cfg.numAttrs = 1;
     }
@@ -1062,7 +1071,7 @@ int verify_common(bool strict, const void* logits, int dtype, int B, int K, int 
   if (reinterpret_cast<uintptr_t>(workspace) % 16 != 0) return ASD_ERR_ALIGN;
   char* ws = static_cast<char*>(workspace);
 
-  VerifyParams p;
+  VerifyParams p = {};
   p.logits = logits;
   p.B = B;
   p.K = K;
@@ -1161,8 +1170,30 @@ int asd_verify_launches(int B, int K, int V, int dtype, int* launches) {
   const int rc = check_shape(B, K, V, dtype);
   if (rc != ASD_OK) return rc;
   const long long request_bytes = static_cast<long long>(K + 1) * V * (dtype_code(dtype) == ASD_BF16 ? 2 : 4);
-  const Path path = choose_path(request_bytes * B, request_bytes, K, true);
-  *launches = B == 0 ? 0 : (path == Path::kTma && use_split() ? 2 : 1);
+  const LaunchOptions opt = launch_options();
+  const Path path = choose_path(opt.path, request_bytes * B, request_bytes, K, true);
+  *launches = B == 0 ? 0 : (path == Path::kTma && opt.split ? 2 : 1);
+  return ASD_OK;
+}
+
+int asd_set_launch_options(const asd_launch_options* options) {
+  if (!options) {
+    g_path.store(ASD_PATH_AUTO);
+    g_flags.store(0);
+    return ASD_OK;
+  }
+  if (options->path < ASD_PATH_AUTO || options->path > ASD_PATH_TMA) return ASD_ERR_CONTROL;
+  g_path.store(options->path);
+  g_flags.store((options->fused_select ? 1 : 0) | (options->no_pdl ? 2 : 0));
+  return ASD_OK;
+}
+
+int asd_get_launch_options(asd_launch_options* options) {
+  if (!options) return ASD_ERR_NULL;
+  const LaunchOptions o = launch_options();
+  options->path = o.path;
+  options->fused_select = o.split ? 0 : 1;
+  options->no_pdl = o.pdl ? 0 : 1;
   return ASD_OK;
 }
 

@@ -18,6 +18,8 @@ What pins what:
   * fp32 gate and budget arithmetic: boundaries built with numpy float32
     division and addition (IEEE, correctly rounded) and one ulp below them;
   * the Fig. 1 worked case: the hand-derived fixture in tests/golden;
+  * ledger validity (NaN or negative budget / spent, spent above the budget):
+    a hand-written table of ledgers and whether each is valid;
   * fused LM-head logits: numpy float64 matmul.
 """
 from __future__ import annotations
@@ -308,6 +310,59 @@ def pin_status_flags(lib):
     assert np.array_equal(res["ledger"][1:], led[1:])
 
 
+# (budget, spent, valid): the ledger rule read from Sec. 3.2-3.3 (a budget is a
+# non-negative amount, the spent regret a non-negative sum of regrets never above
+# it, Eq. 13's invariant s <= B), written out case by case. A negative budget
+# always comes with a negative spent or a spent above it, so that rule needs no
+# test of its own; the table still lists such ledgers.
+LEDGER_TABLE = [
+    (4.0, 0.0, True),
+    (4.0, 4.0, True),           # exhausted: still a valid ledger
+    (4.0, -0.0, True),          # -0 is not below zero
+    (-0.0, 0.0, True),          # zero budget (strict dispatch)
+    (math.inf, 0.0, True),
+    (math.inf, math.inf, True),
+    (math.nan, 0.0, False),     # NaN budget
+    (4.0, math.nan, False),     # NaN spent
+    (math.nan, math.nan, False),
+    (4.0, -1.0, False),         # negative spent
+    (4.0, -math.inf, False),
+    (-1.0, -2.0, False),        # negative budget (and spent)
+    (-math.inf, -math.inf, False),
+    (-1.0, 0.0, False),         # negative budget, spent above it
+    (1.0, 2.0, False),          # spent above the budget
+    (0.0, 1e-30, False),
+]
+
+
+def pin_ledger_validity(lib):
+    """Each ledger of LEDGER_TABLE on a block whose drafts all match: a valid ledger accepts the
+    whole block (a = K, bonus y*_K), an invalid one is flagged, accepts nothing, emits y*_0 and
+    keeps its ledger bit for bit (NaN payloads included)."""
+    B, K, V = len(LEDGER_TABLE), 3, 8
+    z = np.zeros((B, K + 1, V), np.float32)
+    y = (np.arange(B * (K + 1)).reshape(B, K + 1) % (V - 1)) + 1
+    for b in range(B):
+        for j in range(K + 1):
+            z[b, j, y[b, j]] = 5.0
+    x = y[:, :K].astype(np.int32)
+    led = np.array([[bud, sp] for bud, sp, _ in LEDGER_TABLE], np.float32)
+    res = oracle.verify(z, x, led, gate=1.0, cap=2, lib=lib)
+    for b, (bud, sp, valid) in enumerate(LEDGER_TABLE):
+        what = f"ledger ({bud}, {sp})"
+        if valid:
+            assert res["status"][b] == 0, what
+            assert res["accepted_len"][b] == K, what
+            assert res["recovery"][b] == y[b, K], what
+            assert res["ledger"][b, 0] == led[b, 0] and res["ledger"][b, 1] == led[b, 1], what
+        else:
+            assert res["status"][b] == oracle.STATUS_BAD_LEDGER, what
+            assert res["accepted_len"][b] == 0, what
+            assert res["recovery"][b] == y[b, 0], what
+            assert list(res["committed"][b]) == [y[b, 0]] + [-1] * K, what
+            assert np.array_equal(res["ledger"][b].view(np.uint32), led[b].view(np.uint32)), what
+
+
 def pin_lmhead_vs_numpy(lib):
     import torch
     rng = np.random.default_rng(18)
@@ -383,7 +438,7 @@ def pin_commit_fig1(lib):
 
 ALL_PINS = [pin_argmax_vs_numpy, pin_regret_vs_gather, pin_selection_bruteforce, pin_zero_budget_is_strict,
             pin_gate_and_budget_boundaries, pin_fig1, pin_cap_zero_is_strict, pin_carry_ledger,
-            pin_status_flags, pin_lmhead_vs_numpy, pin_select_replays_verify, pin_opportunity_eq4,
+            pin_status_flags, pin_ledger_validity, pin_lmhead_vs_numpy, pin_select_replays_verify, pin_opportunity_eq4,
             pin_commit_fig1]
 
 

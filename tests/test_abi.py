@@ -147,3 +147,27 @@ def test_binding_fails_loudly_without_library(tmp_path):
             mod.load(str(tmp_path / "missing.so"))
         finally:
             importlib.reload(asd)
+
+
+def test_launch_options_round_trip(lib):
+    """asd_set_launch_options / asd_get_launch_options: host-only state, read by every later call."""
+    try:
+        assert asd.get_launch_options() == {"path": "auto", "fused_select": False, "pdl": True}
+        n = ctypes.c_int(-1)
+        assert lib.asd_verify_launches(32, 8, 151936, asd.BF16, ctypes.byref(n)) == 0 and n.value == 2
+        asd.set_launch_options(path="stream", fused_select=True, pdl=False)
+        assert asd.get_launch_options() == {"path": "stream", "fused_select": True, "pdl": False}
+        assert lib.asd_verify_launches(32, 8, 151936, asd.BF16, ctypes.byref(n)) == 0 and n.value == 1
+        asd.set_launch_options(path="tma", fused_select=True)
+        assert lib.asd_verify_launches(4, 8, 1024, asd.F32, ctypes.byref(n)) == 0 and n.value == 1
+        asd.set_launch_options(path="tma")
+        assert lib.asd_verify_launches(4, 8, 1024, asd.F32, ctypes.byref(n)) == 0 and n.value == 2
+
+        class Bad(ctypes.Structure):
+            _fields_ = [("path", ctypes.c_int), ("a", ctypes.c_int), ("b", ctypes.c_int)]
+        assert lib.asd_set_launch_options(ctypes.byref(Bad(7, 0, 0))) == 4  # ASD_ERR_CONTROL
+        assert asd.get_launch_options()["path"] == "tma"  # a rejected call changes nothing
+        assert lib.asd_get_launch_options(None) == 1      # ASD_ERR_NULL
+    finally:
+        asd.reset_launch_options()
+    assert asd.get_launch_options()["path"] == "auto"

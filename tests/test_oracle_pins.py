@@ -51,6 +51,10 @@ def test_status_flags(oracle_lib):
     P.pin_status_flags(oracle_lib)
 
 
+def test_ledger_validity_table(oracle_lib):
+    P.pin_ledger_validity(oracle_lib)
+
+
 def test_lmhead_fp64_matches_numpy(oracle_lib):
     P.pin_lmhead_vs_numpy(oracle_lib)
 
@@ -177,6 +181,13 @@ MUTANTS = {
     "opportunity strict tau": ("if (r[i - 1] <= tau[t]) num[t * np + u] += 1;", "if (r[i - 1] < tau[t]) num[t * np + u] += 1;"),
     "commit drops the recovery token": ("for (int j = 0; j <= a; j++) tokens", "for (int j = 0; j < a; j++) tokens"),
     "commit forgets the pending token": ("if (kv_len) kv_len[b] += pending + a;", "if (kv_len) kv_len[b] += a;"),
+    "ledger check misses a NaN budget": ("if (budget != budget || spent != spent) return 1;",
+                                          "if (spent != spent) return 1;"),
+    "ledger check misses a NaN spent": ("if (budget != budget || spent != spent) return 1;",
+                                         "if (budget != budget) return 1;"),
+    "ledger check accepts a negative spent": ("if (budget < 0.0f || spent < 0.0f) return 1;",
+                                               "if (budget < 0.0f) return 1;"),
+    "bad ledger flagged but still selected": ("if (flags) {\n    a = 0;", "if (flags & ~ORC_STATUS_BAD_LEDGER) {\n    a = 0;"),
     "opportunity suffix starts at i": ("for (int l = i + 1; reusable && l <= i + p[u]; l++)", "for (int l = i; reusable && l < i + p[u]; l++)"),
 }
 
@@ -194,3 +205,20 @@ def test_pins_catch_planted_mistakes(name, tmp_path):
     lib = oracle.load_library(lib_path)
     failed = P.run_all(lib, quick=True)
     assert failed, f"no pin caught the planted mistake: {name}"
+
+
+def test_lmhead_matmul_path_equals_the_loop(oracle_lib):
+    """oracle.lmhead_logits_matmul (numpy float64 matmul over W in blocks of rows) evaluates the same fp64
+    logits as the C loop, across block edges and on integer inputs exactly."""
+    import torch
+    rng = np.random.default_rng(21)
+    T, H, V = 7, 200, 50
+    h = torch.from_numpy(rng.normal(size=(T, H)).astype(np.float32)).to(torch.bfloat16)
+    W = torch.from_numpy(rng.normal(scale=0.02, size=(V, H)).astype(np.float32)).to(torch.bfloat16)
+    z64, _ = oracle.lmhead_logits(h, W, lib=oracle_lib)
+    for block in (8, 13, 64):
+        zm = oracle.lmhead_logits_matmul(h, W, v_block=block)
+        assert np.max(np.abs(zm - z64)) <= 1e-12
+    hi = torch.from_numpy(rng.integers(-1, 2, size=(T, H)).astype(np.float32)).to(torch.bfloat16)
+    Wi = torch.from_numpy(rng.integers(-1, 2, size=(V, H)).astype(np.float32)).to(torch.bfloat16)
+    assert np.array_equal(oracle.lmhead_logits_matmul(hi, Wi, v_block=16), oracle.lmhead_logits(hi, Wi, lib=oracle_lib)[0])

@@ -17,11 +17,12 @@ pytestmark = pytest.mark.gpu
 
 
 @pytest.fixture(params=["stream", "tma", "tma-fused"])
-def kernel(request, monkeypatch):
-    """tma-fused: the TMA row stage with the selection inside it (ASD_VERIFY_SPLIT=0)."""
-    monkeypatch.setenv("ASD_VERIFY_KERNEL", request.param.split("-")[0])
-    monkeypatch.setenv("ASD_VERIFY_SPLIT", "0" if request.param.endswith("fused") else "1")
-    return request.param
+def kernel(request, asd):
+    """tma-fused: the TMA row stage with the selection inside it (last CTA done)."""
+    name = request.param
+    asd.set_launch_options(path=name.split("-")[0], fused_select=name.endswith("fused"))
+    yield name
+    asd.reset_launch_options()
 
 
 def run_sharded(asd, logits, draft, bounds, ledger, gate, cap, misalign=0, resident=False):

@@ -80,3 +80,49 @@ def test_noalloc_rejects_problems_beyond_its_scratch(asd):
     assert rc == SCRATCH_LIMIT
     torch.cuda.synchronize()
     assert int(out["accepted_len"][0]) == -7  # nothing was launched
+
+
+def _same(out_n, out_v, led_n, led_v, what):
+    for key in ("accepted_len", "committed", "recovery", "row_argmax", "status"):
+        assert torch.equal(out_n[key], out_v[key]), f"{what}: {key}"
+    assert np.array_equal(out_n["row_regret"].cpu().numpy().view(np.uint32),
+                          out_v["row_regret"].cpu().numpy().view(np.uint32)), f"{what}: row_regret"
+    assert np.array_equal(led_n.cpu().numpy().view(np.uint32), led_v.cpu().numpy().view(np.uint32)), f"{what}: ledger"
+
+
+def test_noalloc_binding_with_resident_inputs(asd):
+    """The Python binding (asd.verify_noalloc) with ASD_RESIDENT_INPUTS, against asd.verify with the same
+    flag, on two calls in a row of the Qwen3-14B-shaped step."""
+    B, K, V = 32, 8, 151936
+    led_n, led_v = asd.make_ledger(B, 4.0), asd.make_ledger(B, 4.0)
+    ws = asd.Workspace(B, K, V, asd.BF16)
+    for call in range(2):
+        blk = inputs.gen_block(B, K, V, torch.bfloat16, 91_000 + call, "cuda")
+        out_n = asd.verify_noalloc(blk.logits, blk.draft, led_n, 1.0, 2, resident=True)
+        out_v = asd.verify(blk.logits, blk.draft, led_v, 1.0, 2, workspace=ws, resident=True)
+        torch.cuda.synchronize()
+        _same(out_n, out_v, led_n, led_v, f"call {call}")
+
+
+def test_noalloc_at_its_scratch_limit(asd):
+    """The largest batch whose workspace fits ASD_NOALLOC_SCRATCH_BYTES (K=7) runs and matches asd_verify
+    on two calls in a row; the first batch beyond it is rejected before anything is launched."""
+    limit = 1 << 20
+    K, V = 7, 64
+    B = 1
+    while asd.workspace_size(B + 1, K, V, asd.F32) <= limit:  # the largest batch that fits
+        B += 1
+    B_over = B + 1
+    assert asd.workspace_size(B, K, V, asd.F32) <= limit < asd.workspace_size(B_over, K, V, asd.F32)
+    led_n, led_v = asd.make_ledger(B, 4.0), asd.make_ledger(B, 4.0)
+    ws = asd.Workspace(B, K, V, asd.F32)
+    for call in range(2):
+        blk = inputs.gen_block(B, K, V, torch.float32, 92_000 + call, "cuda")
+        out_n = asd.verify_noalloc(blk.logits, blk.draft, led_n, 1.0, 2)
+        out_v = asd.verify(blk.logits, blk.draft, led_v, 1.0, 2, workspace=ws)
+        torch.cuda.synchronize()
+        _same(out_n, out_v, led_n, led_v, f"call {call}")
+    blk = inputs.gen_block(B_over, K, V, torch.float32, 92_100, "cuda")
+    with pytest.raises(asd.AsdError) as err:
+        asd.verify_noalloc(blk.logits, blk.draft, asd.make_ledger(B_over, 4.0), 1.0, 2)
+    assert err.value.code == SCRATCH_LIMIT
