@@ -83,13 +83,11 @@ def recorded_traffic(kernel: str, workload: str | None = None) -> float | None:
     try:
         with open(TRAFFIC_FILE) as f:
             rec = json.load(f)[kernel]
-        if workload is not None:
-            rec = rec["workloads"][workload]
-    except (OSError, ValueError, KeyError, TypeError):
+        if rec.get("sources_sha256") != source_digest(kernel):
+            return None
+        return float(rec["dram_bytes_per_launch"] if workload is None else rec["workloads"][workload])
+    except (OSError, ValueError, KeyError, TypeError, AttributeError):
         return None
-    if rec.get("sources_sha256") != source_digest(kernel):
-        return None
-    return float(rec["dram_bytes_per_launch"])
 
 
 def bf16_peaks() -> dict:
