@@ -453,3 +453,32 @@ def test_zero_budget_is_strict_on_the_large_configs(asd, cfg_id, dtype):
             assert np.array_equal(g[key], s[key]), f"strict entry: {key}"
             assert np.array_equal(g[key], o[key]), f"oracle strict: {key}"
         assert np.array_equal(g["ledger"], np.zeros((B, 2), np.float32))
+
+
+@pytest.mark.parametrize("shape", [(4, 8, 1024, torch.float32), (32, 8, 151936, torch.bfloat16),
+                                   (64, 31, 3000, torch.bfloat16)])
+def test_launches_without_programmatic_dependent_launch(asd, shape):
+    """The no_pdl launch option (plain stream order, no early start) gives the same results bit for bit
+    as the default launches, on each row-stage kernel the shape reaches, over four carried blocks."""
+    B, K, V, dtype = shape
+    blocks = [inputs.gen_block(B, K, V, dtype, 9300 + i, "cuda") for i in range(4)]
+    results = {}
+    try:
+        for pdl in (True, False):
+            for path in ("auto", "stream", "tma"):
+                asd.set_launch_options(path=path, pdl=pdl)
+                led = asd.make_ledger(B, 4.0)
+                outs = [gpu_verify(asd, b.logits, b.draft, led, 1.0, 2) for b in blocks]
+                results[(pdl, path)] = outs
+    finally:
+        asd.reset_launch_options()
+    ref = results[(True, "auto")]
+    for key, outs in results.items():
+        for i, (g, r) in enumerate(zip(outs, ref)):
+            for k in ("accepted_len", "committed", "recovery", "row_argmax", "status", "ledger"):
+                assert np.array_equal(g[k].view(np.uint32) if g[k].dtype == np.float32 else g[k],
+                                      r[k].view(np.uint32) if r[k].dtype == np.float32 else r[k]), \
+                    f"{key} block {i}: {k}"
+    led0 = np.array([[4.0, 0.0]] * B, np.float32)
+    o = oracle.verify(blocks[0].logits.cpu(), blocks[0].draft.cpu().numpy(), led0, 1.0, 2)
+    assert_parity(results[(False, "auto")][0], o, "no pdl, block 0")
