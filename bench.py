@@ -13,6 +13,9 @@ collective on the data path; the barrier and the max over ranks time the job).
 
 --impl reference times the CPU oracle as it stands on the host cores (rank 0
 only), one full block of the same workload per step.
+
+--case NAME --launches N runs only a few launches of one workload (the
+profiler captures in profiles/ use it).
 """
 from __future__ import annotations
 
