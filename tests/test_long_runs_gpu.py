@@ -213,3 +213,33 @@ def test_bench_graph_every_step_matches_oracle(asd, resident):
     for i in range(nsteps):
         check_block(_np(outs[i]), expect[i], f"ledger-history replay step {i}", h[i])
     assert wl.workspace.error() == 0
+
+
+@pytest.mark.parametrize("path", ["auto", "stream"])
+def test_more_than_2_31_logits(asd, path):
+    """B=1600, K=8, V=151936 bf16: 2.19e9 logits (4.4 GB), past every 32-bit element offset. The TMA row
+    stage (with and without resident inputs) and the register-streaming kernel match the oracle, which
+    runs request slices in parallel (requests are independent; each slice carries its own ledgers)."""
+    B, K, V = 1600, 8, 151936
+    assert B * (K + 1) * V > 2**31
+    b = inputs.gen_block(B, K, V, torch.bfloat16, 7_777, "cuda")
+    led0 = np.array([[4.0, 0.0]] * B, np.float32)
+    outs = []
+    try:
+        asd.set_launch_options(path=path)
+        for resident in (False, True):
+            led = torch.from_numpy(led0.copy()).cuda()
+            out = _np(asd.verify(b.logits, b.draft, led, 1.0, 2, resident=resident))
+            out["ledger"] = led.cpu().numpy()
+            outs.append(out)
+    finally:
+        asd.reset_launch_options()
+    z, x = b.logits.cpu(), b.draft.cpu().numpy()
+    del b
+    step = 100
+    with cf.ThreadPoolExecutor(max_workers=16) as pool:
+        parts = list(pool.map(lambda s: oracle.verify(z[s:s + step], x[s:s + step], led0[s:s + step], 1.0, 2),
+                              range(0, B, step)))
+    o = {k: np.concatenate([p[k] for p in parts]) for k in parts[0]}
+    for g in outs:
+        check_block(g, o, f"{path} > 2^31 logits", g["ledger"])
