@@ -478,7 +478,8 @@ def run_gpu(args) -> None:
     clocks.stop()
     timed = clocks.window(clocks.t0, clocks.t1)
     if timed["sm_mhz"] is not None:
-        clk = dict(timed, window="timed region")
+        clk = dict(timed, window="the timed region and 0.25 s either side of it (one sample every 200 ms; the "
+                                 "step graph ran back to back over the 1 s before it)")
     else:
         clk = dict(clocks.window(t_soak, clocks.t1),
                    window="1 s of the same step graph ending at the timed region (which is shorter than "
