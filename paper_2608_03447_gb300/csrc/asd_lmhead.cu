@@ -30,7 +30,6 @@
 #include <stdint.h>
 
 #include <atomic>
-#include <cstdlib>
 #include <mutex>
 
 #include "asd.h"

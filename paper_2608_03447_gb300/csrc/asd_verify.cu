@@ -1,29 +1,31 @@
 // libasd: verifier of Approximate Speculative Decoding (arXiv 2608.03447) for
-// GB300 (sm_103a). Logit-streaming path: asd_verify / asd_verify_strict.
+// GB300 (sm_103a). Logit-streaming path: asd_verify, asd_verify_strict,
+// asd_verify_blocks, asd_shard_partials and asd_verify_noalloc.
 //
-// One launch does the whole step:
-//   stage 1  row reduction (Eq. 1, Eq. 3). The [B, K+1, V] logits are treated
-//            as one flat array and cut into equal, 16-byte aligned ranges, one
-//            per warp, so every SM streams the same number of bytes whatever
-//            B, K and V are. A warp walks its range row segment by row
-//            segment with 128-bit streaming loads, keeps a per-lane running
-//            maximum (NaN-propagating, so a NaN cannot hide), and reduces the
-//            segment to one 64-bit key (order-preserving fp32 bits, then the
-//            inverted vocabulary index) that one atomicMax merges into the
-//            row's slot: the largest key is the largest logit at the lowest
-//            index, whatever order the segments finish in. The segment that
-//            holds the draft token also records z_j(x_j).
-//   stage 2  selection (Eq. 5-13, Alg. 1). Each warp adds the element count
-//            it finished to its request's counter; the warp that completes a
-//            request runs the request's selection with lane j owning target
-//            row j, and resets the request's workspace slots to zero, so that
-//            the whole workspace is zero again after every call (whatever
-//            shape the next call has).
+// A step is two stages over the [B, K+1, V] logits, treated as one flat array:
+//   row stage  (Eq. 1, Eq. 3) the flat array is cut into equal, 16-byte
+//              aligned ranges; each range is streamed with 128-bit loads (or
+//              TMA bulk copies into a shared-memory ring), every lane keeps a
+//              NaN-propagating running maximum, and each row segment reduces
+//              to one 64-bit key (order-preserving fp32 bits, then the
+//              inverted vocabulary index) merged into the row's slot by
+//              atomicMax: the largest key is the largest logit at the lowest
+//              index, whatever order the segments finish in. The segment that
+//              holds the draft token also records z_j(x_j).
+//   selection  (Eq. 5-13, Alg. 1) one warp per request, lane j owning target
+//              row j, resets the request's workspace slots to zero as it reads
+//              them, so the workspace is zero again after every call (whatever
+//              shape the next call has).
+// Three row-stage kernels cover the input sizes: verify_small_kernel (one CTA
+// per request, selection in the same CTA) below 1 MB when a request fits one
+// round of loads, verify_kernel (register streaming; the warp that completes a
+// request selects it) for other small inputs, and verify_tma_kernel from 1 MB,
+// followed by select_kernel (or, as a launch option, selecting in the CTA that
+// completes each request).
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
-#include <cstdlib>
 #include <atomic>
 #include <mutex>
 
