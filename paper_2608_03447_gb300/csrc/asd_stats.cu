@@ -2,12 +2,13 @@
 //
 // Over every draft-target mismatch position (x, i) of the given blocks, count
 // those whose regret is at most tau and that are followed, inside the block,
-// by p draft tokens equal to the target's argmax; also count |M|. One thread
-// per block-request works on bit masks of the K positions: m (x_j == y*_j),
-// d = ~m, R_t (r_j <= tau_t) and S_p = AND_{k=1..p} (m >> k) (the next p
-// tokens match; bits past the block are zero, which also enforces i + p <= K),
-// then counts with popc. A CTA sums its threads in shared memory and adds to
-// the caller's counters once per counter.
+// by p draft tokens equal to the target's argmax; also count |M|. One warp per
+// block-request: lane j loads position j (one round of loads for the whole
+// block), and ballots give the bit masks m (x_j == y*_j), d = ~m and
+// R_t (r_j <= tau_t); S_p = AND_{k=1..p} (m >> k) (the next p tokens match;
+// bits past the block are zero, which also enforces i + p <= K). Lanes then
+// split the counters and count with popc. A CTA sums its warps in shared
+// memory and adds to the caller's counters once per counter.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -22,43 +23,53 @@ struct OpportunityArgs {
 };
 
 constexpr int kStatThreads = 256;
+constexpr int kStatWarps = kStatThreads / 32;
+constexpr unsigned kFullMask = 0xffffffffu;
 
-__global__ void __launch_bounds__(kStatThreads) opportunity_kernel(const int32_t* __restrict__ row_argmax,
-                                                                   const int32_t* __restrict__ draft,
-                                                                   const float* __restrict__ row_regret,
-                                                                   const int32_t* __restrict__ status, int n, int K,
-                                                                   const OpportunityArgs a,
-                                                                   unsigned long long* counts) {
+__global__ void __launch_bounds__(kStatThreads)
+    opportunity_kernel(const int32_t* __restrict__ row_argmax, const int32_t* __restrict__ draft,
+                       const float* __restrict__ row_regret, const int32_t* __restrict__ status, int n, int K,
+                       const __grid_constant__ OpportunityArgs a, unsigned long long* counts) {
   __shared__ unsigned int local[ASD_OPPORTUNITY_MAX * ASD_OPPORTUNITY_MAX + 1];
+  __shared__ uint32_t s_mask[kStatWarps][2 * ASD_OPPORTUNITY_MAX];  // S_p per p, then R_t per tau
   const int ncount = a.ntau * a.np;
   for (int i = threadIdx.x; i <= ncount; i += blockDim.x) local[i] = 0u;
   __syncthreads();
 
-  const int b = blockIdx.x * blockDim.x + threadIdx.x;
-  if (b < n && !(status && status[b] != 0)) {
-    const int32_t* y = row_argmax + static_cast<long long>(b) * (K + 1);
-    const int32_t* x = draft + static_cast<long long>(b) * K;
-    const float* r = row_regret + static_cast<long long>(b) * K;
-    uint32_t m = 0;
-    uint32_t rmask[ASD_OPPORTUNITY_MAX];
-    for (int t = 0; t < a.ntau; ++t) rmask[t] = 0u;
-    for (int j = 0; j < K; ++j) {
-      if (x[j] == y[j]) m |= 1u << j;
-      const float rj = r[j];
-      for (int t = 0; t < a.ntau; ++t)
-        if (rj <= a.tau[t]) rmask[t] |= 1u << j;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const long long b = static_cast<long long>(blockIdx.x) * kStatWarps + warp;
+  if (b < n) {  // warp-uniform
+    // every load of the block-request at once, the status included
+    const bool mine = lane < K;
+    int xj = 0, yj = 0;
+    float rj = 0.0f;
+    if (mine) {
+      xj = draft[b * K + lane];
+      yj = row_argmax[b * (K + 1) + lane];
+      rj = row_regret[b * K + lane];
     }
-    const uint32_t all = K >= 32 ? 0xffffffffu : ((1u << K) - 1u);
-    const uint32_t d = ~m & all;  // M restricted to this block
-    if (d) atomicAdd(&local[ncount], static_cast<unsigned>(__popc(d)));
-    for (int u = 0; u < a.np; ++u) {
-      uint32_t s = all;
-      for (int k = 1; k <= a.p[u] && s; ++k) s &= m >> k;
-      const uint32_t e = d & s;
-      if (!e) continue;
-      for (int t = 0; t < a.ntau; ++t) {
-        const int c = __popc(e & rmask[t]);
-        if (c) atomicAdd(&local[t * a.np + u], static_cast<unsigned>(c));
+    const int st = status ? status[b] : 0;
+    if (st == 0) {
+      const uint32_t m = __ballot_sync(kFullMask, mine && xj == yj);
+      const uint32_t all = K >= 32 ? 0xffffffffu : ((1u << K) - 1u);
+      const uint32_t d = ~m & all;  // M restricted to this block
+      if (d) {
+        for (int t = 0; t < a.ntau; ++t) {
+          const uint32_t r = __ballot_sync(kFullMask, mine && rj <= a.tau[t]);
+          if (lane == t) s_mask[warp][ASD_OPPORTUNITY_MAX + t] = r;
+        }
+        if (lane < a.np) {
+          uint32_t sp = all;
+          for (int k = 1; k <= a.p[lane] && sp; ++k) sp &= m >> k;
+          s_mask[warp][lane] = sp;
+        }
+        __syncwarp();
+        for (int c = lane; c < ncount; c += 32) {
+          const int t = c / a.np, u = c - t * a.np;
+          const int cnt = __popc(d & s_mask[warp][u] & s_mask[warp][ASD_OPPORTUNITY_MAX + t]);
+          if (cnt) atomicAdd(&local[c], static_cast<unsigned>(cnt));
+        }
+        if (lane == 0) atomicAdd(&local[ncount], static_cast<unsigned>(__popc(d)));
       }
     }
   }
@@ -88,7 +99,7 @@ extern "C" int asd_opportunity(const int32_t* row_argmax, const int32_t* draft, 
   }
   if (n == 0 || K == 0) return ASD_OK;  // no position can mismatch
   if (!row_argmax || !draft || !row_regret) return ASD_ERR_NULL;
-  const unsigned grid = static_cast<unsigned>((n + kStatThreads - 1) / kStatThreads);
+  const unsigned grid = static_cast<unsigned>((n + kStatWarps - 1) / kStatWarps);
   opportunity_kernel<<<grid, kStatThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
       row_argmax, draft, row_regret, status, n, K, a, counts);
   return cudaGetLastError() == cudaSuccess ? ASD_OK : ASD_ERR_CUDA;
