@@ -134,6 +134,18 @@ def run_lmhead(dev, clocks=None, iters: int = 20, sustain_s: float = 1.2) -> dic
     torch.cuda.synchronize(dev)
     ms, tb0, tb1 = timed(iters)
     flop = 2.0 * LM_B * (LM_K + 1) * LM_H * LM_V
+    # the library GEMM of the same shape alone (bf16 logits out, no reduction), timed the same way
+    logits = torch.empty(LM_B * (LM_K + 1), LM_V, dtype=torch.bfloat16, device=dev)
+    for _ in range(3):
+        torch.matmul(inp.hidden, inp.weight.t(), out=logits)
+    c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    c0.record(stream)
+    for _ in range(iters):
+        torch.matmul(inp.hidden, inp.weight.t(), out=logits)
+    c1.record(stream)
+    c1.synchronize()
+    ms_gemm = c0.elapsed_time(c1) / iters
+    del logits
     tflops = flop / (ms * 1e-3) / 1e12
     pk = bf16_peaks()
     # one of four tensor-parallel ranks: its quarter of W, the partials (the all-gather and the
@@ -166,7 +178,7 @@ def run_lmhead(dev, clocks=None, iters: int = 20, sustain_s: float = 1.2) -> dic
         return None if c.get("sm_mhz") is None else t * c["sm_mhz"] / 1e3
 
     summary = {"bound": "tensor", "achieved": tflops, "peak": pk["burst"], "unit": "TFLOP/s",
-               "frac": tflops / pk["burst"], "ms": ms, "sm_mhz": clk_b.get("sm_mhz"),
+               "frac": tflops / pk["burst"], "ms": ms, "library_gemm_ms": ms_gemm, "sm_mhz": clk_b.get("sm_mhz"),
                "ms_x_ghz": ghz_ms(ms, clk_b),
                "sustained": {"ms": ms_sus, "achieved": tflops_sus, "peak": pk["sustained"],
                              "frac": tflops_sus / pk["sustained"], "sm_mhz": clk_s.get("sm_mhz"),
@@ -802,11 +814,15 @@ def run_case(name: str, launches: int) -> None:
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
     asd.load()
-    if name == "lmhead":
+    if name in ("lmhead", "cublas-lmhead"):
         inp = inputs.gen_lmhead(LM_B, LM_K, LM_H, LM_V, inputs.seed_for(4), dev)
         led = asd.make_ledger(LM_B, 8.0, 0.0, dev)
+        logits = torch.empty(LM_B * (LM_K + 1), LM_V, dtype=torch.bfloat16, device=dev)
         for _ in range(2 + launches):
-            asd.lmhead_verify(inp.hidden, inp.weight, inp.draft, led, 1.0, 2)
+            if name == "lmhead":
+                asd.lmhead_verify(inp.hidden, inp.weight, inp.draft, led, 1.0, 2)
+            else:  # the library GEMM of the same shape (bf16 logits out, no reduction), for comparison
+                torch.matmul(inp.hidden, inp.weight.t(), out=logits)
         torch.cuda.synchronize(dev)
         print(json.dumps({"case": name, "launches": 2 + launches}))
         return
@@ -835,7 +851,7 @@ def main():
     ap.add_argument("--impl", default="asd", choices=["asd", "reference"])
     ap.add_argument("--case", default=None,
                     help="run only a few launches of one workload (for ncu): " + ", ".join(
-                        list(CASES) + ["lmhead"] + [f"torch-amax:{c}" for c in CASES]))
+                        list(CASES) + ["lmhead", "cublas-lmhead"] + [f"torch-amax:{c}" for c in CASES]))
     ap.add_argument("--launches", type=int, default=3)
     ap.add_argument("--no-configs", dest="configs", action="store_false",
                     help="skip timing the other workloads (configs 0, 2, 3)")

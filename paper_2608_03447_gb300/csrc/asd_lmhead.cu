@@ -7,23 +7,27 @@
 // token's logit, with no [T, V] logit buffer); the selection of Alg. 1 then
 // runs as in asd_verify. The logits never reach global memory.
 //
-// Tiling: two CTAs on a pair of SMs (a cluster of 2) share one 2-SM MMA
-// (tcgen05 cta_group::2). The MMA's M is 256 vocabulary rows (128 per SM:
-// the TMEM lanes), its N is 192 token rows (the TMEM columns); each SM loads
-// its own 128 rows of W and half (96) of the token rows, so an SM takes in
-// 28 KB of operands per 64-deep K step for a 128 x 192 x 64 product, and the
-// 576 rows of a B = 64, K = 8 step are exactly three token tiles (no padded
-// rows). A pair owns one token tile and walks the vocabulary tiles with a
-// stride; the pairs of the three token tiles that share a vocabulary tile run
-// at the same time, so each W tile comes from HBM once and from L2 for the
-// other two. Per CTA: warp 0 issues TMA loads (128B-swizzled 64-wide K slabs)
-// into a kStages-deep ring, whose completion is counted on the first CTA's
-// barrier; warp 1 allocates tensor memory, and in the first CTA one of its
-// threads issues the MMAs; warps 2-5 read the accumulator with tcgen05.ld.
-// The 512 TMEM columns hold two 192-column accumulators, so the epilogue of
-// one vocabulary tile overlaps the MMAs of the next. The epilogue reduces
-// each token column over the 32 vocabulary rows of a warp with a transposing
-// butterfly of (value, index) keys and keeps a running key per token.
+// Tiling: two CTAs on a pair of SMs (a cluster of 2) share 2-SM MMAs
+// (tcgen05 cta_group::2). An MMA's M is 256 vocabulary rows (128 per SM: the
+// TMEM lanes), its N is 192 token rows (the TMEM columns), and the 576 rows of
+// a B = 64, K = 8 step are exactly three token tiles (no padded rows). A pair
+// works in units of two vocabulary tiles (512 rows) against one token tile:
+// per 64-deep K step each SM loads 256 rows of W and half (96) of the token
+// rows, 44 KB, and issues two MMAs over the same token slab, so the token rows
+// cross from L2 once per two vocabulary tiles. A pair owns one token tile and
+// walks the units with a stride; the pairs of the three token tiles that share
+// a unit run at the same time, so each W tile comes from HBM once and from L2
+// for the other two. Per CTA: warp 0 issues TMA loads (128B-swizzled 64-wide K
+// slabs) into a kStages-deep ring, whose completion is counted on the first
+// CTA's barrier; warp 1 allocates tensor memory, and in the first CTA one of
+// its threads issues the MMAs; warps 2-9 read the two accumulators (192 of the
+// 512 TMEM columns each) with tcgen05.ld, one warp per lane quarter and tile.
+// The epilogue turns each 32 x 32 block (vocabulary rows x token columns) of a
+// warp around through shared memory, so that a lane holds one token column and
+// reduces it with plain register arithmetic, and keeps a running (value, index)
+// key per token. The MMAs of the next unit wait for the epilogue: two
+// accumulators fill the tensor memory, and this costs less than the extra L2
+// traffic of one vocabulary tile per unit with double-buffered accumulators.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -39,34 +43,38 @@ namespace {
 
 using namespace asd_detail;
 
-constexpr int kPairM = 256;               // vocabulary rows per CTA pair (MMA M)
-constexpr int kHalfM = 128;               // vocabulary rows per CTA (TMEM lanes)
+constexpr int kPairM = 256;               // vocabulary rows per CTA pair in one MMA (MMA M)
+constexpr int kHalfM = 128;               // vocabulary rows per CTA in one MMA (TMEM lanes)
 constexpr int kTN = 192;                  // token rows per tile (MMA N)
 constexpr int kHalfN = kTN / 2;           // token rows each CTA of the pair loads
 constexpr int kBK = 64;                   // K per stage: 64 bf16 = one 128-byte swizzle row
 constexpr int kUmmaK = 16;                // K per tcgen05.mma (kind::f16)
-#ifndef ASD_LM_STAGES
-#define ASD_LM_STAGES 7
-#endif
-constexpr int kStages = ASD_LM_STAGES;
+constexpr int kW = 2;                     // vocabulary tiles per unit (MMAs per token slab)
+constexpr int kUnitM = kW * kPairM;       // vocabulary rows per pair per unit
+constexpr int kStages = 4;
 constexpr int kStageB = kHalfN * kBK * 2;  // 12 KB of token rows
-constexpr int kStageA = kHalfM * kBK * 2;  // 16 KB of vocabulary rows
+constexpr int kSlabA = kHalfM * kBK * 2;   // 16 KB of vocabulary rows per tile
+constexpr int kStageA = kW * kSlabA;
 constexpr uint32_t kStageTx = 2u * (kStageA + kStageB);  // both CTAs' bytes, counted on the first CTA
-constexpr int kLmThreads = 6 * 32;        // producer, MMA, 4 epilogue warps
-constexpr int kTmemCols = 512;            // two accumulators at columns 0 and 256
+constexpr int kEpiWarps = 4 * kW;         // one per TMEM lane quarter and vocabulary tile
+constexpr int kLmThreads = (2 + kEpiWarps) * 32;  // producer, MMA, epilogue warps
+constexpr int kTmemCols = 512;            // accumulator j at column j * 256
 constexpr int kAccStride = 256;
 constexpr int kChunks = kTN / 32;         // 32-column TMEM loads per accumulator
+constexpr int kPitch = 36;                // floats per row of an epilogue transpose block (conflict-free)
 static_assert(kTN % 32 == 0 && kHalfN % 8 == 0, "token tile: whole 32-column loads, whole 8-row swizzle groups");
+static_assert((kW - 1) * kAccStride + kTN <= kTmemCols, "accumulators fit in tensor memory");
 
 struct LmShared {
   unsigned long long full[kStages];   // first CTA: both CTAs' loads of a stage have landed
   unsigned long long empty[kStages];  // each CTA: the MMAs have read its part of a stage
-  unsigned long long acc_full[2];     // each CTA: an accumulator is complete
-  unsigned long long acc_empty[2];    // first CTA: both CTAs' epilogues have read an accumulator
+  unsigned long long acc_full;        // each CTA: the unit's accumulators are complete
+  unsigned long long acc_empty;       // first CTA: both CTAs' epilogues have read them
   unsigned long long drain;
   uint32_t tmem_base;
   int abort;
   int draft[kTN];                     // x of the tile's token rows (-1: no draft / out of range)
+  alignas(16) float xpose[kEpiWarps][32 * kPitch];  // per epilogue warp: a 32 x 32 block turned around
 };
 // dynamic shared memory: [1 KB alignment slack][stages x B][stages x A][LmShared]
 constexpr size_t kLmSmemBytes = 1024 + static_cast<size_t>(kStages) * (kStageA + kStageB) + sizeof(LmShared);
@@ -211,36 +219,17 @@ __device__ __forceinline__ void abort_pair(LmShared& sh, uint32_t peer) {
 // whatever its sign bit, so a NaN anywhere in a row reaches the row's key.
 __device__ __forceinline__ uint32_t max_bits(float v) { return v != v ? 0xffc00000u : ordered_bits(v); }
 
-// Warp-wide transposing maximum: lane l holds the logits of its vocabulary
-// row for 32 token columns (z[0..31]); afterwards lane l holds, in z[0], the
-// maximum over the 32 lanes of column l (NaN if any of them is NaN). Five
-// exchange levels; at each the lane keeps the half of its columns selected
-// by its lane bit and receives the partner's values for that half.
-__device__ __forceinline__ float transpose_max32(float (&z)[32], int lane) {
-#pragma unroll
-  for (int half = 16; half >= 1; half >>= 1) {
-    const bool up = (lane & half) != 0;
-#pragma unroll
-    for (int i = 0; i < half; ++i) {
-      const float send = up ? z[i] : z[i + half];
-      const float keep = up ? z[i + half] : z[i];
-      z[i] = fmax_nan(keep, __shfl_xor_sync(kFull, send, half));
-    }
-  }
-  return z[0];
-}
-
 struct LmParams {
   int T, H, V;
   int token_tiles;     // ceil(T / kTN)
   int pairs_per_tile;  // CTA pairs that share one token tile
-  int vocab_tiles;     // ceil(V / kPairM)
+  int vocab_units;     // ceil(V / kUnitM)
   int k_steps;         // ceil(H / kBK)
   float* logits_out;   // [T, V] when writing logits instead of verifying
 };
 
 // One CTA pair (cluster of 2): token tile m = pair % token_tiles, vocabulary
-// tiles n = pair / token_tiles + i * pairs_per_tile.
+// units n = pair / token_tiles + i * pairs_per_tile (rows n * kUnitM on).
 template <bool kStrict, bool kWriteLogits>
 __global__ void __launch_bounds__(kLmThreads, 1)
     lmhead_verify_kernel(const __grid_constant__ CUtensorMap map_h, const __grid_constant__ CUtensorMap map_w,
@@ -261,7 +250,7 @@ __global__ void __launch_bounds__(kLmThreads, 1)
   const int m = pair % q.token_tiles;
   const int n_first = pair / q.token_tiles;
   const int n_tiles =
-      n_first < q.vocab_tiles ? (q.vocab_tiles - n_first + q.pairs_per_tile - 1) / q.pairs_per_tile : 0;
+      n_first < q.vocab_units ? (q.vocab_units - n_first + q.pairs_per_tile - 1) / q.pairs_per_tile : 0;
   const int K1 = p.K + 1;
 
   if (threadIdx.x == 0) {
@@ -269,10 +258,8 @@ __global__ void __launch_bounds__(kLmThreads, 1)
       mbar_init(&sh.full[s], 1);
       mbar_init(&sh.empty[s], 1);
     }
-    for (int a = 0; a < 2; ++a) {
-      mbar_init(&sh.acc_full[a], 1);
-      mbar_init(&sh.acc_empty[a], 8);  // 4 epilogue warps in each CTA
-    }
+    mbar_init(&sh.acc_full, 1);
+    mbar_init(&sh.acc_empty, 2 * kEpiWarps);  // the epilogue warps of both CTAs
     mbar_init(&sh.drain, 1);
     sh.abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -322,7 +309,8 @@ __global__ void __launch_bounds__(kLmThreads, 1)
           if (leader) mbar_expect_tx(&sh.full[s], kStageTx);
           const uint32_t bar = full0 + static_cast<uint32_t>(s * sizeof(unsigned long long));
           tma_load_2d_pair(sB + s * kStageB, &map_h, bar, k * kBK, m * kTN + static_cast<int>(rank) * kHalfN);
-          tma_load_2d_pair(sA + s * kStageA, &map_w, bar, k * kBK, n * kPairM + static_cast<int>(rank) * kHalfM);
+          // this CTA's 128 rows of both vocabulary tiles of the unit: rows n * 512 + rank * 256 on
+          tma_load_2d_pair(sA + s * kStageA, &map_w, bar, k * kBK, n * kUnitM + static_cast<int>(rank) * kW * kHalfM);
           it_issued = it + 1;
         }
       }
@@ -332,14 +320,13 @@ __global__ void __launch_bounds__(kLmThreads, 1)
     if (leader && lane == 0) {
       int it = 0;
       for (int t = 0; t < n_tiles && !sh.abort; ++t) {
-        const int a = t & 1;
-        if (!mbar_wait_cluster(&sh.acc_empty[a], ((t >> 1) & 1) ^ 1, &sh.abort)) {
+        // the epilogues of both CTAs have read the previous unit's accumulators
+        if (!mbar_wait_cluster(&sh.acc_empty, (t & 1) ^ 1, &sh.abort)) {
           abort_pair(sh, peer);
           report_timeout(p);
           break;
         }
         tc_fence_after();
-        const uint32_t d = tmem + static_cast<uint32_t>(a * kAccStride);
         bool ok = true;
         for (int k = 0; k < q.k_steps; ++k, ++it) {
           const int s = it % kStages;
@@ -348,12 +335,16 @@ __global__ void __launch_bounds__(kLmThreads, 1)
             break;
           }
           tc_fence_after();
-          const uint64_t ad = smem_desc_sw128(sA + s * kStageA);
           const uint64_t bd = smem_desc_sw128(sB + s * kStageB);
 #pragma unroll
-          for (int kk = 0; kk < kBK / kUmmaK; ++kk) {
-            // advance 16 elements (32 bytes, encoded 2) along K inside the swizzle row
-            umma_pair_bf16(d, ad + 2u * kk, bd + 2u * kk, (k > 0 || kk > 0) ? 1u : 0u);
+          for (int j = 0; j < kW; ++j) {  // both vocabulary tiles of the unit read the same token slab
+            const uint32_t d = tmem + static_cast<uint32_t>(j * kAccStride);
+            const uint64_t ad = smem_desc_sw128(sA + s * kStageA + j * kSlabA);
+#pragma unroll
+            for (int kk = 0; kk < kBK / kUmmaK; ++kk) {
+              // advance 16 elements (32 bytes, encoded 2) along K inside the swizzle row
+              umma_pair_bf16(d, ad + 2u * kk, bd + 2u * kk, (k > 0 || kk > 0) ? 1u : 0u);
+            }
           }
           umma_commit_pair(&sh.empty[s]);  // frees the stage in both CTAs when these MMAs have read it
         }
@@ -362,7 +353,7 @@ __global__ void __launch_bounds__(kLmThreads, 1)
           report_timeout(p);
           break;
         }
-        umma_commit_pair(&sh.acc_full[a]);  // the accumulator is complete in both CTAs
+        umma_commit_pair(&sh.acc_full);  // the accumulators are complete in both CTAs
       }
       umma_commit_local(&sh.drain);  // arrives once every MMA issued above has finished
       const unsigned long long t0 = global_ns();
@@ -370,10 +361,13 @@ __global__ void __launch_bounds__(kLmThreads, 1)
       }
     }
   } else {
-    // ---------------- epilogue: warps 2-5, one vocabulary row (TMEM lane) per thread
+    // ---------------- epilogue: warps 2 .. 1 + kEpiWarps, one vocabulary row (TMEM lane) per thread;
+    // warps 2-5 read the first vocabulary tile of a unit, warps 6-9 the second
     const int quarter = warp & 3;                     // TMEM lanes this warp may read
+    const int jt = (warp - 2) >> 2;                   // the unit's vocabulary tile this warp reduces
     const uint32_t lane_base = static_cast<uint32_t>(quarter * 32) << 16;
-    const uint32_t acc_empty0 = map_rank(smem_u32(&sh.acc_empty[0]), 0);
+    const uint32_t acc_empty0 = map_rank(smem_u32(&sh.acc_empty), 0);
+    float* xpose = sh.xpose[warp - 2];
     int xs[kChunks];  // lane l: draft of token column c * 32 + l
 #pragma unroll
     for (int c = 0; c < kChunks; ++c) xs[c] = kWriteLogits ? -1 : sh.draft[c * 32 + lane];
@@ -381,8 +375,7 @@ __global__ void __launch_bounds__(kLmThreads, 1)
 #pragma unroll
     for (int c = 0; c < kChunks; ++c) best[c] = 0ull;
     for (int t = 0; t < n_tiles; ++t) {
-      const int a = t & 1;
-      const bool ok = __all_sync(kFull, mbar_wait_cluster(&sh.acc_full[a], (t >> 1) & 1, &sh.abort));
+      const bool ok = __all_sync(kFull, mbar_wait_cluster(&sh.acc_full, t & 1, &sh.abort));
       if (!ok) {
         if (lane == 0) {
           abort_pair(sh, peer);
@@ -391,12 +384,13 @@ __global__ void __launch_bounds__(kLmThreads, 1)
         break;
       }
       tc_fence_after();
-      const int v_warp = (n_first + t * q.pairs_per_tile) * kPairM + static_cast<int>(rank) * kHalfM + quarter * 32;
+      const int v_warp = (n_first + t * q.pairs_per_tile) * kUnitM + static_cast<int>(rank) * kW * kHalfM +
+                         jt * kHalfM + quarter * 32;
       const int v = v_warp + lane;  // this thread's vocabulary row
 #pragma unroll
       for (int c = 0; c < kChunks; ++c) {
         uint32_t r[32];
-        tmem_ld32(tmem + lane_base + static_cast<uint32_t>(a * kAccStride + c * 32), r);
+        tmem_ld32(tmem + lane_base + static_cast<uint32_t>(jt * kAccStride + c * 32), r);
         tmem_ld_wait();
         if (kWriteLogits) {
           if (v < q.V) {
@@ -421,42 +415,40 @@ __global__ void __launch_bounds__(kLmThreads, 1)
               p.draft_logit[m * kTN + c * 32 + i] = z;
             }
           }
-          // argmax of each column over the warp's 32 rows: the maximum by a
-          // transposing butterfly, then, for the columns whose running maximum
-          // it raises, the lowest row holding it (a ballot of equal values).
+          // argmax of each column over the warp's 32 rows: the block is turned
+          // around through shared memory (lane l writes its row, then reads
+          // column l), the lane takes the column's maximum, and where that
+          // raises the column's running key, the lowest row holding it.
           if (v_warp >= q.V) continue;  // rows past the vocabulary: nothing to reduce
-          float z[32];
+          if (v_warp + 31 >= q.V && v >= q.V) {  // the last, partial tile: rows past V never win
 #pragma unroll
-          for (int i = 0; i < 32; ++i) z[i] = __uint_as_float(r[i]);
-          if (v_warp + 31 >= q.V) {  // the last, partial tile: rows past V never win
-#pragma unroll
-            for (int i = 0; i < 32; ++i)
-              if (v >= q.V) z[i] = -INFINITY;
+            for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(-INFINITY);
           }
-          const float zmax = transpose_max32(z, lane);
-          const uint32_t hi = max_bits(zmax);
-          const unsigned raise = __ballot_sync(kFull, hi > static_cast<uint32_t>(best[c] >> 32));
-          if (raise) {
-            unsigned rows = 0;  // lane l: rows of column l that hold its maximum
 #pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              if ((raise >> i) & 1u) {
-                const float zi = __shfl_sync(kFull, zmax, i);
-                const float mine = v < q.V ? __uint_as_float(r[i]) : -INFINITY;
-                const unsigned eq = __ballot_sync(kFull, mine == zi);
-                if (lane == i) rows = eq;
-              }
-            }
-            if ((raise >> lane) & 1u) {
-              const int w = rows ? __ffs(rows) - 1 : 0;  // NaN: no row compares equal; the key still says NaN
-              best[c] = (static_cast<unsigned long long>(hi) << 32) | (0xffffffffu - static_cast<uint32_t>(v_warp + w));
-            }
+          for (int i = 0; i < 8; ++i)
+            *reinterpret_cast<uint4*>(xpose + lane * kPitch + 4 * i) =
+                make_uint4(r[4 * i], r[4 * i + 1], r[4 * i + 2], r[4 * i + 3]);
+          __syncwarp();
+          float col[32];  // column `lane` of the block: the logits of token c * 32 + lane in the warp's 32 rows
+#pragma unroll
+          for (int i = 0; i < 32; ++i) col[i] = xpose[i * kPitch + lane];
+          __syncwarp();  // the block is read before the next chunk overwrites it
+          float zmax = col[0];
+#pragma unroll
+          for (int i = 1; i < 32; ++i) zmax = fmax_nan(zmax, col[i]);
+          const uint32_t hi = max_bits(zmax);
+          if (hi > static_cast<uint32_t>(best[c] >> 32)) {
+            int w = 0;  // NaN: no row compares equal; the key still says NaN
+#pragma unroll
+            for (int i = 31; i >= 0; --i)
+              if (col[i] == zmax) w = i;
+            best[c] = (static_cast<unsigned long long>(hi) << 32) | (0xffffffffu - static_cast<uint32_t>(v_warp + w));
           }
         }
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive_remote(acc_empty0 + static_cast<uint32_t>(a * sizeof(unsigned long long)));
+      if (lane == 0) mbar_arrive_remote(acc_empty0);
     }
     if (!kWriteLogits && !sh.abort) {
 #pragma unroll
@@ -600,15 +592,15 @@ int launch_lmhead(const void* hidden, const void* weight, int H, int T, VerifyPa
     dev->pairs[slot].store(pairs, std::memory_order_release);
   }
   CUtensorMap map_h, map_w;
-  if (!make_map(&map_h, hidden, T, H, kHalfN) || !make_map(&map_w, weight, p.V, H, kHalfM)) return ASD_ERR_CUDA;
+  if (!make_map(&map_h, hidden, T, H, kHalfN) || !make_map(&map_w, weight, p.V, H, kW * kHalfM)) return ASD_ERR_CUDA;
   LmParams q;
   q.T = T;
   q.H = H;
   q.V = p.V;
   q.token_tiles = (T + kTN - 1) / kTN;
   q.pairs_per_tile = pairs / q.token_tiles > 0 ? pairs / q.token_tiles : 1;
-  q.vocab_tiles = (p.V + kPairM - 1) / kPairM;
-  if (q.pairs_per_tile > q.vocab_tiles) q.pairs_per_tile = q.vocab_tiles;
+  q.vocab_units = (p.V + kUnitM - 1) / kUnitM;
+  if (q.pairs_per_tile > q.vocab_units) q.pairs_per_tile = q.vocab_units;
   q.k_steps = (H + kBK - 1) / kBK;
   q.logits_out = logits_out;
   const unsigned grid = 2u * static_cast<unsigned>(q.token_tiles * q.pairs_per_tile);
