@@ -310,6 +310,36 @@ def test_lmhead_sharded_partials_combine_to_the_unsharded_verify(asd, B, K, H, V
     assert np.array_equal(led_s.cpu().numpy().view(np.int32), o["ledger"].view(np.int32))
 
 
+def test_lmhead_full_size_four_shards_equal_the_unsharded_verify(asd):
+    """B=64, K=8, H=5120, V=151936 on integer h and W, the vocabulary cut into the four 37984-row shards
+    of four tensor-parallel ranks (each shard ends inside a 512-row unit): the combined partials equal
+    the unsharded fused verify bit for bit (that one equals the oracle on these inputs, above)."""
+    cfg = inputs.CONFIGS[4]
+    B, K, H, V = cfg["B"], cfg["K"], cfg["H"], cfg["V"]
+    inp = inputs.gen_lmhead_exact(B, K, H, V, inputs.seed_for(4, 1), "cuda")
+    T = B * (K + 1)
+    S = 4
+    bounds = [i * V // S for i in range(S + 1)]
+    parts = torch.empty(S, T, asd.PARTIAL_WORDS, dtype=torch.int32, device="cuda")
+    for i in range(S):
+        shard = inp.weight[bounds[i]:bounds[i + 1]].contiguous()
+        asd.lmhead_partials(inp.hidden, shard, inp.draft, bounds[i], V, out=parts[i])
+        del shard
+    led_s = asd.make_ledger(B, cfg["budget"])
+    sharded = asd.shard_combine(parts, inp.draft, led_s, cfg["gate"], cfg["cap"], V)
+    led_u = asd.make_ledger(B, cfg["budget"])
+    whole = asd.lmhead_verify(inp.hidden, inp.weight, inp.draft, led_u, cfg["gate"], cfg["cap"])
+    torch.cuda.synchronize()
+    for key in ("accepted_len", "committed", "recovery", "row_argmax", "status"):
+        assert np.array_equal(sharded[key].cpu().numpy(), whole[key].cpu().numpy()), key
+    assert np.array_equal(sharded["row_regret"].cpu().numpy().view(np.int32),
+                          whole["row_regret"].cpu().numpy().view(np.int32))
+    assert np.array_equal(led_s.cpu().numpy().view(np.int32), led_u.cpu().numpy().view(np.int32))
+    # the winners are spread over the shards, so the combine had real work to do
+    owner = np.searchsorted(np.array(bounds[1:]), whole["row_argmax"].cpu().numpy().reshape(-1), side="right")
+    assert len(set(owner.tolist())) == S
+
+
 def test_lmhead_verify_infinities_through_the_tensor_cores(asd):
     """A +inf weight: where h is +1 the row's logit is +inf (it wins), where h is -1 it is -inf, and
     0 x inf = NaN flags the request; every other output equals the fp64 oracle (IEEE on both sides)."""
