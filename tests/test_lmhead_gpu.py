@@ -224,7 +224,7 @@ def test_lmhead_full_size_exact_inputs_bit_exact(asd):
 
 
 @pytest.mark.parametrize("B,K,H,V", [(8, 8, 512, 1000), (40, 8, 256, 2100), (5, 0, 64, 777), (3, 16, 320, 1300),
-                                     (1500, 9, 64, 300)])
+                                     (1500, 9, 64, 300), (6, 8, 8, 1000), (7, 3, 40, 513)])
 def test_lmhead_verify_exact_inputs_bit_exact(asd, B, K, H, V):
     """Integer h and W: the fp32 logits are exact, so every output equals the oracle's bit for bit,
     ties across warps, SMs and SM pairs included (lowest index wins)."""
