@@ -192,7 +192,7 @@ int asd_verify_strict(const void* logits, int dtype, int B, int K, int V, const 
  * order, so ties and near-ties (within about 1e-5 of the row's scale) may
  * resolve differently from an exact (fp64) evaluation; exact ties between
  * equal fp32 logits go to the lowest index, as in asd_verify.
- * Launch: clusters of two CTAs, one per SM of a pair, each with about 200 KB
+ * Launch: clusters of two CTAs, one per SM of a pair, each with about 214 KB
  * of shared memory and all 512 tensor-memory columns of its SM, so a call
  * occupies the GPU's SM pairs while it runs.
  */
