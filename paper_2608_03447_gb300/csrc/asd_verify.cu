@@ -667,19 +667,10 @@ __global__ void __launch_bounds__(kTmaThreads, ASD_TMA_MIN_BLOCKS)
   const int nchunks = lo < hi ? static_cast<int>((hi - lo + kChunkElems - 1) / kChunkElems) : 0;
 
   pdl_signal_dependents();
-  // Unless the caller declared the inputs resident, the previous kernel on the
-  // stream may be the one writing them: read nothing before it has completed.
-  if (!p.resident) pdl_wait_prerequisites();
 
-  // each consumer's first row is known now: start its draft-id load before the
-  // first copy lands
-  RowCursor c;
-  c.next_x = -1;
-  const long long first_a = lo + static_cast<long long>(warp) * kWarpElems;
-  const bool head_here = blockIdx.x == 0 && warp == 0 && p.head > 0;
-  if (warp < kTmaConsumers) c.next_x = draft_of_row(p, head_here ? 0 : (first_a < hi ? first_a : 0) / p.V);
-
-  // this CTA's rows, including the ragged head (CTA 0) and tail (last CTA)
+  // Shared-memory set-up first: it reads no input, so a launch that has to
+  // wait for the previous kernel does it while waiting.
+  // This CTA's rows, including the ragged head (CTA 0) and tail (last CTA).
   const long long cta_lo = blockIdx.x == 0 ? 0 : lo;
   const long long cta_hi = blockIdx.x == gridDim.x - 1 ? p.total : hi;
   RowSink sink;
@@ -691,7 +682,6 @@ __global__ void __launch_bounds__(kTmaThreads, ASD_TMA_MIN_BLOCKS)
     sh.row_key[t] = 0ull;
     sh.row_bits[t] = 0u;
   }
-
   if (threadIdx.x == 0) {
     for (int s = 0; s < kTmaStages; ++s) {
       mbar_init(&sh.full[s], 1);
@@ -702,6 +692,18 @@ __global__ void __launch_bounds__(kTmaThreads, ASD_TMA_MIN_BLOCKS)
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
   __syncthreads();
+
+  // Unless the caller declared the inputs resident, the previous kernel on the
+  // stream may be the one writing them: read nothing before it has completed.
+  if (!p.resident) pdl_wait_prerequisites();
+
+  // each consumer's first row is known now: start its draft-id load before the
+  // first copy lands
+  RowCursor c;
+  c.next_x = -1;
+  const long long first_a = lo + static_cast<long long>(warp) * kWarpElems;
+  const bool head_here = blockIdx.x == 0 && warp == 0 && p.head > 0;
+  if (warp < kTmaConsumers) c.next_x = draft_of_row(p, head_here ? 0 : (first_a < hi ? first_a : 0) / p.V);
 
   int issued = 0;  // producer: chunks issued
   if (warp == kTmaConsumers) {
