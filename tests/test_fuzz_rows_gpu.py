@@ -90,7 +90,7 @@ def test_random_fused_lmhead_exact_inputs(asd, chunk):
         B = int(rng.choice([1, 2, 7, 21, 64]))
         K = int(rng.choice([0, 1, 5, 8, 16]))
         H = int(rng.choice([8, 64, 136, 512, 1032]))
-        V = int(rng.choice([1, 255, 256, 257, 700, 3001]))
+        V = int(rng.choice([1, 255, 256, 257, 511, 512, 513, 700, 1025, 3001]))
         inp = inputs.gen_lmhead_exact(B, K, H, V, 45_000 + chunk * 100 + i, "cuda")
         led0 = np.array([[8.0, 0.0]] * B, np.float32)
         led = torch.from_numpy(led0.copy()).cuda()
