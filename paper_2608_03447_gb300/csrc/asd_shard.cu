@@ -12,6 +12,7 @@
 
 #include "asd.h"
 #include "asd_device.cuh"
+#include "asd_launch.cuh"
 
 namespace {
 
@@ -25,6 +26,8 @@ __global__ void __launch_bounds__(kCombineThreads) shard_combine_kernel(const as
   const int warps = blockDim.x / 32;
   const int K = p.K, K1 = p.K + 1;
   const long long R = static_cast<long long>(p.B) * K1;
+  pdl_signal_dependents();
+  pdl_wait_prerequisites();  // the partials are read only once the kernel before this one is done
   for (int b = blockIdx.x * warps + (threadIdx.x >> 5); b < p.B; b += gridDim.x * warps) {
     BlockInputs in;
     in.key = 0ull;
@@ -97,6 +100,9 @@ extern "C" int asd_shard_combine(const asd_partial* partials, int S, int B, int 
   p.status = status;
   constexpr int kWarps = kCombineThreads / 32;
   const unsigned grid = static_cast<unsigned>((B + kWarps - 1) / kWarps);
-  shard_combine_kernel<<<grid, kCombineThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(partials, S, p);
+  cudaLaunchAttribute attr;
+  const cudaLaunchConfig_t cfg =
+      pdl_config(dim3(grid), dim3(kCombineThreads), reinterpret_cast<cudaStream_t>(stream), &attr);
+  if (cudaLaunchKernelEx(&cfg, shard_combine_kernel, partials, S, p) != cudaSuccess) return ASD_ERR_CUDA;
   return cudaGetLastError() == cudaSuccess ? ASD_OK : ASD_ERR_CUDA;
 }

@@ -13,8 +13,12 @@
 #include <stdint.h>
 
 #include "asd.h"
+#include "asd_device.cuh"
+#include "asd_launch.cuh"
 
 namespace {
+
+using namespace asd_detail;
 
 struct OpportunityArgs {
   float tau[ASD_OPPORTUNITY_MAX];
@@ -34,6 +38,10 @@ __global__ void __launch_bounds__(kStatThreads)
   __shared__ uint32_t s_mask[kStatWarps][2 * ASD_OPPORTUNITY_MAX];  // S_p per p, then R_t per tau
   const int ncount = a.ntau * a.np;
   for (int i = threadIdx.x; i <= ncount; i += blockDim.x) local[i] = 0u;
+  // programmatic dependent launch: the next kernel may start its set-up now;
+  // this one reads the verify outputs only once the kernel before it is done
+  pdl_signal_dependents();
+  pdl_wait_prerequisites();
   __syncthreads();
 
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -100,8 +108,12 @@ extern "C" int asd_opportunity(const int32_t* row_argmax, const int32_t* draft, 
   if (n == 0 || K == 0) return ASD_OK;  // no position can mismatch
   if (!row_argmax || !draft || !row_regret) return ASD_ERR_NULL;
   const unsigned grid = static_cast<unsigned>((n + kStatWarps - 1) / kStatWarps);
-  opportunity_kernel<<<grid, kStatThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
-      row_argmax, draft, row_regret, status, n, K, a, counts);
+  cudaLaunchAttribute attr;
+  const cudaLaunchConfig_t cfg =
+      pdl_config(dim3(grid), dim3(kStatThreads), reinterpret_cast<cudaStream_t>(stream), &attr);
+  if (cudaLaunchKernelEx(&cfg, opportunity_kernel, row_argmax, draft, row_regret, status, n, K, a, counts) !=
+      cudaSuccess)
+    return ASD_ERR_CUDA;
   return cudaGetLastError() == cudaSuccess ? ASD_OK : ASD_ERR_CUDA;
 }
 
@@ -146,6 +158,8 @@ extern "C" int asd_commit(int B, int K, const int32_t* accepted_len, const int32
   if (B == 0) return ASD_OK;
   if (!accepted_len || !committed) return ASD_ERR_NULL;
   if (tokens && (!token_len || max_tokens < 1)) return ASD_ERR_NULL;
+  // a plain launch: with programmatic dependent launch it measured slower
+  // behind a kernel that does not trigger its dependents early
   constexpr int kWarps = kCommitThreads / 32;
   commit_kernel<<<static_cast<unsigned>((B + kWarps - 1) / kWarps), kCommitThreads, 0,
                   reinterpret_cast<cudaStream_t>(stream)>>>(B, K, accepted_len, committed, pending, kv_len, tokens,
