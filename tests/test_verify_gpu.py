@@ -482,3 +482,59 @@ def test_launches_without_programmatic_dependent_launch(asd, shape):
     led0 = np.array([[4.0, 0.0]] * B, np.float32)
     o = oracle.verify(blocks[0].logits.cpu(), blocks[0].draft.cpu().numpy(), led0, 1.0, 2)
     assert_parity(results[(False, "auto")][0], o, "no pdl, block 0")
+
+
+def test_concurrent_streams_keep_their_own_state(asd):
+    """Three streams issue dependent sequences at the same time, interleaved call by call and never
+    synchronised with each other: the TMA row stage with its selection kernel (Qwen3-14B shape), the
+    one-CTA-per-request kernel (the tiny shape), and the fused LM-head verify (exact inputs). Each
+    stream has its own workspace and ledger; every call equals the oracle, so no call sees another
+    stream's state."""
+    n = 5
+    specs = [(32, 8, 151936, torch.bfloat16), (4, 8, 1024, torch.float32)]
+    seqs = []
+    for s, (B, K, V, dtype) in enumerate(specs):
+        blocks = [inputs.gen_block(B, K, V, dtype, 9400 + 10 * s + i, "cuda") for i in range(n)]
+        led = np.array([[4.0, 0.0]] * B, np.float32)
+        expect = []
+        for b in blocks:
+            o = oracle.verify(b.logits.cpu(), b.draft.cpu().numpy(), led, 1.0, 2)
+            expect.append(o)
+            led = o["ledger"]
+        seqs.append(dict(blocks=blocks, expect=expect, ledger=asd.make_ledger(B, 4.0),
+                         ws=asd.Workspace(B, K, V, asd.BF16 if dtype == torch.bfloat16 else asd.F32),
+                         outs=[asd.alloc_outputs(B, K) for _ in range(n)], stream=torch.cuda.Stream()))
+    Bl, Kl, Hl, Vl = 8, 8, 256, 1300
+    lm = [inputs.gen_lmhead_exact(Bl, Kl, Hl, Vl, 9500 + i, "cuda") for i in range(n)]
+    lm_expect, led = [], np.array([[8.0, 0.0]] * Bl, np.float32)
+    for inp in lm:
+        z64 = oracle.lmhead_logits_matmul(inp.hidden.cpu(), inp.weight.cpu())
+        o = oracle.verify(z64.astype(np.float32).reshape(Bl, Kl + 1, Vl), inp.draft.cpu().numpy(), led, 1.0, 2)
+        lm_expect.append(o)
+        led = o["ledger"]
+    lm_led = asd.make_ledger(Bl, 8.0)
+    lm_ws = asd.lmhead_workspace(Bl, Kl, Vl, Hl, torch.device("cuda"))
+    lm_outs = [asd.alloc_outputs(Bl, Kl) for _ in range(n)]
+    lm_stream = torch.cuda.Stream()
+    for st in [q["stream"] for q in seqs] + [lm_stream]:
+        st.wait_stream(torch.cuda.current_stream())
+    for i in range(n):
+        for q in seqs:
+            with torch.cuda.stream(q["stream"]):
+                b = q["blocks"][i]
+                asd.verify(b.logits, b.draft, q["ledger"], 1.0, 2, workspace=q["ws"], out=q["outs"][i])
+        with torch.cuda.stream(lm_stream):
+            asd.lmhead_verify(lm[i].hidden, lm[i].weight, lm[i].draft, lm_led, 1.0, 2, workspace=lm_ws,
+                              out=lm_outs[i])
+    torch.cuda.synchronize()
+    for s, q in enumerate(seqs):
+        for i in range(n):
+            g = _np(q["outs"][i])
+            for key in ("accepted_len", "committed", "recovery", "row_argmax", "status"):
+                assert np.array_equal(g[key], q["expect"][i][key]), f"stream {s} call {i}: {key}"
+        assert np.array_equal(q["ledger"].cpu().numpy().view(np.int32), q["expect"][-1]["ledger"].view(np.int32))
+    for i in range(n):
+        g = _np(lm_outs[i])
+        for key in ("accepted_len", "committed", "recovery", "row_argmax", "status"):
+            assert np.array_equal(g[key], lm_expect[i][key]), f"LM-head stream call {i}: {key}"
+    assert np.array_equal(lm_led.cpu().numpy().view(np.int32), lm_expect[-1]["ledger"].view(np.int32))
